@@ -1,0 +1,433 @@
+#!/usr/bin/env python
+"""Prefix-KV retrieval benchmark on GB300 (fast tier -> paged GPU KV cache).
+
+Default workload: Llama-3-8B-shaped KV (32 layers, 8 KV heads, head_dim 128,
+bf16, 128 KiB/token), 16 requests of 4096-token prompts at 50% prefix hit
+(2048 matched tokens each, 8 chunks of 256 tokens), 20,000-block paged cache
+with a seeded random block assignment, chunks in pinned host memory.  One step
+= one kvs_retrieve of the whole batch (4 GiB of KV).
+
+Prints ONE JSON line.  ``--impl reference`` times the CPU oracle instead (the
+plain element loop, on the host cores), on the same workload.
+"""
+from __future__ import annotations
+
+import argparse
+import hashlib
+import json
+import os
+import statistics
+import subprocess
+import sys
+import threading
+import time
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+if ROOT not in sys.path:
+    sys.path.insert(0, ROOT)
+
+METRIC = "prefix-KV retrieval GB/s and tokens/s on 1 GB300; % of HBM / host-link roofline"
+MEASURED_PEAKS = os.path.join(ROOT, "MEASURED_PEAKS.json")
+TRAFFIC_FILE = os.path.join(ROOT, "profiles", "traffic.json")
+KERNEL_SRC = os.path.join(ROOT, "paper_2609_35065_gb300", "csrc", "kvs_kernels.cu")
+HBM_FALLBACK_GBS = 6800.0
+
+
+def parse_args(argv=None):
+    ap = argparse.ArgumentParser(description=__doc__.splitlines()[0])
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=50)
+    ap.add_argument("--warmup", type=int, default=5)
+    ap.add_argument("--impl", choices=["ours", "reference"], default="ours")
+    ap.add_argument("--config", default="llama8b",
+                    help="llama8b | sweep25 | sweep50 | sweep75 | qwen14b | llama70b[_25|_50|_100]")
+    ap.add_argument("--variant", choices=["auto", "hostlink", "hbmcopy"], default="auto")
+    ap.add_argument("--kernel", choices=["auto", "ldg", "tma"], default="auto")
+    ap.add_argument("--max-ctas", type=int, default=0)
+    ap.add_argument("--probe-bytes", type=int, default=1 << 30)
+    ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--overlap", action="store_true", help="llama70b: retrieval beside a bf16 GEMM loop")
+    return ap.parse_args(argv)
+
+
+# ---------------------------------------------------------------------------
+def workload(name: str):
+    from paper_2609_35065_gb300 import synth
+    if name == "llama8b":
+        return synth.llama8b()
+    if name.startswith("sweep"):
+        return synth.sweep(int(name[5:]) / 100.0)
+    if name == "qwen14b":
+        return synth.qwen14b()
+    if name.startswith("llama70b"):
+        frac = int(name.split("_")[1]) / 100.0 if "_" in name else 1.0
+        return synth.llama70b(buffer_frac=frac)
+    if name == "tiny":
+        return synth.tiny()
+    raise SystemExit(f"unknown config {name}")
+
+
+def describe(w) -> str:
+    g = w.geom
+    m = w.matched_tokens
+    return (f"{w.name}: L{g.layers} H{g.kv_heads} D{g.head_dim} bf16 B{g.block_size} C{g.chunk_tokens}, "
+            f"{len(w.requests)} requests, {m} matched tokens, NB {w.num_blocks}")
+
+
+def token_bytes(g) -> int:
+    return 2 * g.layers * g.row_elems * g.elem_bytes
+
+
+def measured_peaks() -> dict:
+    try:
+        with open(MEASURED_PEAKS) as f:
+            return json.load(f)
+    except (OSError, ValueError):
+        return {}
+
+
+def kernel_hash() -> str:
+    with open(KERNEL_SRC, "rb") as f:
+        return hashlib.sha256(f.read()).hexdigest()[:16]
+
+
+def recorded_traffic(kernel: str, config: str):
+    """Per-launch DRAM bytes from an ncu capture of the current kernel source, else None."""
+    try:
+        with open(TRAFFIC_FILE) as f:
+            rec = json.load(f)
+    except (OSError, ValueError):
+        return None
+    ent = rec.get(f"{config}/{kernel}")
+    if not ent or ent.get("kernel_sha") != kernel_hash():
+        return None
+    return ent.get("dram_bytes_per_launch")
+
+
+class ClockSampler:
+    """nvidia-smi clocks and throttle reasons, timestamped on arrival."""
+    FIELDS = ("clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+              "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+              "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, index: int):
+        self.samples = []
+        self.proc = None
+        try:
+            self.proc = subprocess.Popen(
+                ["nvidia-smi", "-i", str(index), f"--query-gpu={self.FIELDS}", "--format=csv,noheader,nounits",
+                 "-lms", "50"], stdout=subprocess.PIPE, stderr=subprocess.DEVNULL, text=True)
+        except OSError:
+            return
+        self.thread = threading.Thread(target=self._read, daemon=True)
+        self.thread.start()
+
+    def _read(self):
+        for line in self.proc.stdout:
+            self.samples.append((time.time(), [x.strip() for x in line.split(",")]))
+
+    def stop(self):
+        if self.proc:
+            self.proc.terminate()
+            try:
+                self.proc.wait(timeout=5)
+            except subprocess.TimeoutExpired:
+                self.proc.kill()
+
+    def summary(self, t0: float, t1: float):
+        if not self.samples:
+            return None
+        inside = [s for t, s in self.samples if t0 - 0.06 <= t <= t1 + 0.06] or \
+                 [min(self.samples, key=lambda ts: abs(ts[0] - (t0 + t1) / 2))[1]]
+        names = ("hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap")
+        reasons = set()
+        sm, mx = [], []
+        for s in inside:
+            try:
+                sm.append(float(s[0]))
+                mx.append(float(s[1]))
+            except (ValueError, IndexError):
+                continue
+            for k, nm in enumerate(names):
+                if len(s) > 4 + k and s[4 + k].lower().startswith("active"):
+                    reasons.add(nm)
+        if not sm:
+            return None
+        return {"sm_mhz": statistics.median(sm), "sm_max_mhz": max(mx), "reasons": sorted(reasons),
+                "samples": len(sm)}
+
+
+# ---------------------------------------------------------------------------
+# CPU oracle (baseline / reference arm)
+# ---------------------------------------------------------------------------
+def oracle_inputs_from_buffers(buf):
+    from paper_2609_35065_gb300.buffers import NP_DTYPES
+    npd = NP_DTYPES[buf.workload.geom.elem_bytes]
+    return [[(t.numpy() if t.device.type == "cpu" else t.cpu().numpy()).view(npd) for t in mine]
+            for mine in buf.chunks]
+
+
+def oracle_pass(w, chunks_np, threads: int, planes=None) -> float:
+    """One pass of the workload through the CPU oracle (planes [lo, hi) or all);
+    each thread owns one reusable host plane.  Returns seconds."""
+    import numpy as np
+    from concurrent.futures import ThreadPoolExecutor
+    import oracle
+
+    g = w.geom
+    P = 2 * g.layers
+    planes = list(range(P)) if planes is None else list(planes)
+    n = w.num_blocks * g.block_size * g.row_elems
+    local = threading.local()
+
+    def one(p):
+        buf = getattr(local, "buf", None)
+        if buf is None:
+            buf = local.buf = np.empty(n, dtype=np.uint16)
+        ps = [None] * P
+        ps[p] = buf
+        for r, req in enumerate(w.requests):
+            if chunks_np[r]:
+                oracle.retrieve(g.layers, g.kv_heads, g.head_dim, g.block_size, ps, w.num_blocks,
+                                req.first_token, chunks_np[r], req.block_table, p0=p, p1=p + 1)
+
+    with ThreadPoolExecutor(threads) as ex:
+        list(ex.map(lambda p: None, range(threads)))     # start threads before timing
+        t = time.perf_counter()
+        list(ex.map(one, planes))
+        return time.perf_counter() - t
+
+
+def cpu_chunks(w):
+    """Chunk buffers of ``w`` on the host (seeded, torch CPU generator)."""
+    import numpy as np
+    import torch
+    from paper_2609_35065_gb300 import buffers
+    buf = buffers.allocate(w, device="cpu", with_planes=False)
+    return [[t.numpy().view(np.uint16) for t in mine] for mine in buf.chunks]
+
+
+def host_cores() -> int:
+    return len(os.sched_getaffinity(0))
+
+
+def run_reference(args):
+    rank = int(os.environ.get("RANK", "0"))
+    if rank != 0:
+        return 0
+    w = workload(args.config)
+    chunks_np = cpu_chunks(w)
+    cores = host_cores()
+    payload = w.matched_tokens * token_bytes(w.geom)
+    for _ in range(args.warmup):
+        oracle_pass(w, chunks_np, cores)
+    total = 0.0
+    for _ in range(args.steps):
+        total += oracle_pass(w, chunks_np, cores)
+    gbs = payload * args.steps / total / 1e9
+    line = {
+        "metric": METRIC, "value": round(gbs, 3), "unit": "GB/s", "impl": "reference",
+        "n_gpus": args.gpus, "steps": args.steps, "warmup": args.warmup,
+        "ms_per_step": round(total / args.steps * 1e3, 3), "higher_is_better": True,
+        "scaling": "weak", "vs_baseline": None, "dtype": "bf16 (copied as u16)", "data": "synthetic",
+        "config": {"workload": describe(w), "source": "host memory (oracle reads numpy buffers)"},
+        "tokens_per_s": round(w.matched_tokens * args.steps / total, 1),
+        "cpu_baseline": {"value": round(gbs, 3), "unit": "GB/s", "cores": cores, "kind": "oracle",
+                         "sample": f"every step = the whole workload ({payload} bytes), all {2 * w.geom.layers} planes"},
+        "e2e": {"value": round(gbs, 3), "unit": "GB/s", "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},
+    }
+    print(json.dumps(line), flush=True)
+    return 0
+
+
+# ---------------------------------------------------------------------------
+# GPU arm
+# ---------------------------------------------------------------------------
+def run_ours(args):
+    import numpy as np
+    import torch
+    from paper_2609_35065_gb300 import buffers, kvs
+
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    rank = int(os.environ.get("RANK", "0"))
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    dist = None
+    if world > 1:
+        import torch.distributed as dist
+        torch.cuda.set_device(local)
+        dist.init_process_group("nccl")
+    else:
+        torch.cuda.set_device(0)
+    dev = torch.cuda.current_device()
+
+    def barrier():
+        if dist is not None:
+            dist.barrier()
+        torch.cuda.synchronize()
+
+    kvs.lib()
+    stream = torch.cuda.Stream()
+    bw = kvs.kvs_query_bw(stream, args.probe_bytes)
+    host_peak = max(bw["h2d_copy_engine_gbs"], bw["zero_copy_read_gbs"])
+
+    w = workload(args.config)
+    g = w.geom
+    buf = buffers.allocate(w)
+    payload = buf.payload_bytes
+    tokens = w.matched_tokens
+    flags = 0
+    if args.variant == "hostlink":
+        flags |= kvs.KVS_F_FORCE_HOSTLINK
+    elif args.variant == "hbmcopy":
+        flags |= kvs.KVS_F_FORCE_HBMCOPY
+    if args.kernel == "ldg":
+        flags |= kvs.KVS_F_FORCE_LDG
+    elif args.kernel == "tma":
+        flags |= kvs.KVS_F_FORCE_TMA
+    if args.max_ctas:
+        flags |= kvs.KVS_F_MAX_CTAS(args.max_ctas)
+    choice = kvs.kvs_get_choice()
+    host_variant = {"hostlink": 1, "hbmcopy": 2}.get(args.variant, choice["chosen_retrieve_host"])
+
+    def step(requests, f=flags):
+        kvs.kvs_retrieve(g, buf.plane_ptrs, w.num_blocks, requests, stream, f)
+
+    # correctness gate before timing: one validated call
+    step(buf.requests, flags | kvs.KVS_F_VALIDATE)
+    for _ in range(args.warmup):
+        step(buf.requests)
+    barrier()
+
+    sampler = ClockSampler(dev)
+    time.sleep(0.15)
+    K = args.steps
+    ev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)) for _ in range(K)]
+    t_start, t_end = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    launches0 = kvs.kvs_stat_launches()
+    barrier()
+    wall0 = time.time()
+    t_start.record(stream)
+    for k in range(K):
+        ev[k][0].record(stream)
+        step(buf.requests)
+        ev[k][1].record(stream)
+    t_end.record(stream)
+    torch.cuda.synchronize()
+    wall1 = time.time()
+    barrier()
+    launches = kvs.kvs_stat_launches() - launches0
+    time.sleep(0.1)
+    sampler.stop()
+    total_ms = t_start.elapsed_time(t_end)
+    if dist is not None:
+        t = torch.tensor([total_ms], device="cuda")
+        dist.all_reduce(t, op=dist.ReduceOp.MAX)
+        total_ms = float(t.item())
+    per_call_ms = [a.elapsed_time(b) for a, b in ev]
+    call_ms = statistics.mean(per_call_ms)
+    value = payload * K * world / (total_ms / 1e3) / 1e9
+    tokens_per_s = tokens * K * world / (total_ms / 1e3)
+    achieved = payload / (call_ms / 1e3) / 1e9
+    kernel_name = "kvs_ldg_kernel" if host_variant == 1 else "hbmcopy_pipeline"
+
+    # e2e: the public API from host arguments, result status read back every step
+    e2e_steps = max(3, min(K, 20))
+    desc_bytes = 8 * 2 * g.layers + sum(len(r.chunks) * (16 + 4 * (g.chunk_tokens // g.block_size))
+                                        for r in buf.requests)
+    barrier()
+    t0 = time.perf_counter()
+    for _ in range(e2e_steps):
+        reqs = [kvs.RequestArg(r.block_table, r.chunks, r.first_token) for r in buf.requests]
+        kvs.kvs_retrieve(g, buf.plane_ptrs, w.num_blocks, reqs, stream, flags)
+        kvs.kvs_check_errors(stream)                      # 4-byte device->host read, synchronises
+    e2e_s = (time.perf_counter() - t0) / e2e_steps
+    e2e = {"value": round(payload * world / e2e_s / 1e9, 3), "unit": "GB/s",
+           "h2d_bytes_per_step": int(payload + desc_bytes), "d2h_bytes_per_step": 4,
+           "ms_per_step": round(e2e_s * 1e3, 3)}
+
+    # device-resident (HBM staging) source, same workload: the HBM roofline
+    hbm = None
+    if rank == 0 and w.name in ("llama8b",):
+        dpool = torch.empty_like(buf.host_pool, device="cuda")
+        dpool.copy_(buf.host_pool)
+        per_tok = 2 * g.layers * g.row_elems
+        dreqs = []
+        at = 0
+        for r in buf.requests:
+            cs = []
+            for c in r.chunks:
+                cs.append(kvs.ChunkArg(dpool[at:at + c.num_tokens * per_tok], c.num_tokens, kvs.KVS_SRC_DEVICE))
+                at += c.num_tokens * per_tok
+            dreqs.append(kvs.RequestArg(r.block_table, cs, r.first_token))
+        dflags = flags & ~(kvs.KVS_F_FORCE_HOSTLINK | kvs.KVS_F_FORCE_HBMCOPY)
+        step(dreqs, dflags | kvs.KVS_F_VALIDATE)
+        for _ in range(3):
+            step(dreqs, dflags)
+        torch.cuda.synchronize()
+        dev_ms = []
+        for _ in range(max(5, min(K, 20))):
+            a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+            a.record(stream)
+            step(dreqs, dflags)
+            b.record(stream)
+            b.synchronize()
+            dev_ms.append(a.elapsed_time(b))
+        dms = statistics.mean(dev_ms)
+        peaks = measured_peaks()
+        hpk = peaks.get("hbm_gbs", HBM_FALLBACK_GBS)
+        ach = 2 * payload / (dms / 1e3) / 1e9
+        kname = "kvs_tma_kernel" if choice["chosen_kernel_device"] == 2 else "kvs_ldg_kernel"
+        hbm = {"bound": "hbm", "achieved": round(ach, 1), "peak": hpk, "unit": "GB/s",
+               "frac": round(ach / hpk, 4), "traffic": recorded_traffic(kname, "llama8b_device"),
+               "kernel": kname, "payload_gbs": round(payload / (dms / 1e3) / 1e9, 1),
+               "peak_source": "MEASURED_PEAKS.json hbm_gbs (copy, read+write bytes)" if peaks else "fallback",
+               "bytes_counted": "2 x payload (read + write)"}
+        del dpool
+
+    cpu = None
+    if rank == 0 and world == 1 and not args.no_cpu_baseline:
+        chunks_np = oracle_inputs_from_buffers(buf)
+        cores = host_cores()
+        secs = oracle_pass(w, chunks_np, cores)
+        cpu = {"value": round(payload / secs / 1e9, 3), "unit": "GB/s", "cores": cores, "kind": "oracle",
+               "sample": f"one full pass of the workload ({payload} bytes, all {2 * g.layers} planes), "
+                         f"threads split by plane"}
+
+    clocks = sampler.summary(wall0, wall1)
+    if rank == 0:
+        line = {
+            "metric": METRIC, "value": round(value, 3), "unit": "GB/s", "n_gpus": world, "steps": K,
+            "warmup": args.warmup, "ms_per_step": round(total_ms / K, 4), "higher_is_better": True,
+            "scaling": "weak", "vs_baseline": None, "dtype": "bf16 (copied as u16)", "data": "synthetic",
+            "config": {"workload": describe(w), "source": "pinned host memory (fast-tier stand-in)",
+                       "variant": {1: "hostlink", 2: "hbmcopy"}[host_variant],
+                       "l2": f"inputs ({payload >> 20} MiB per step) larger than L2; no flush",
+                       "parallelism": f"replicas x{world}"},
+            "tokens_per_s": round(tokens_per_s, 1),
+            "roofline": {"bound": "host_link", "achieved": round(achieved, 2), "peak": round(host_peak, 2),
+                         "unit": "GB/s", "frac": round(achieved / host_peak, 4),
+                         "traffic": recorded_traffic(kernel_name, "llama8b"), "kernel": kernel_name,
+                         "peak_source": "measured in this run: max(copy-engine pinned H2D, zero-copy read kernel)",
+                         "bytes_counted": "payload over the host link"},
+            "roofline_hbm": hbm,
+            "cpu_baseline": cpu,
+            "e2e": e2e,
+            "gpu_launches": int(launches),
+            "clocks": clocks,
+            "bw_probe": {k: (round(v, 2) if isinstance(v, float) else v) for k, v in bw.items()},
+        }
+        print(json.dumps(line), flush=True)
+    if dist is not None:
+        dist.destroy_process_group()
+    return 0
+
+
+def main(argv=None):
+    args = parse_args(argv)
+    if args.impl == "reference":
+        return run_reference(args)
+    return run_ours(args)
+
+
+if __name__ == "__main__":
+    sys.exit(main())

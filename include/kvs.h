@@ -1,0 +1,220 @@
+/*
+ * kvs.h -- C ABI for prefix-KV retrieval into a paged GPU KV cache (GB300, sm_103a).
+ *
+ * TempoKV separates SSD-to-fast-tier staging from fast-tier-to-GPU retrieval
+ * (Sec. 2.2) and reuses the runtime's GPU-transfer path once matched KV is
+ * stage-ready (Sec. 3, Sec. 4).  This library is that transfer path:
+ *
+ *   kvs_retrieve  copies the matched prefix of each request from its chunk
+ *                 buffers in the fast tier into the runtime's paged KV cache;
+ *   kvs_store     copies newly computed KV from the paged cache back into
+ *                 chunk buffers (KV is retained in complete 256-token chunks,
+ *                 Sec. 5.1, Workload);
+ *   kvs_query_bw  measures the host link and HBM on this GPU and picks, per
+ *                 direction, how host-resident chunks are moved.
+ *
+ * The arguments follow the paper's statement of a retrieval: the matched
+ * prefix tokens of each request, where its KV objects sit in the fast tier
+ * (their ordered manifest, Sec. 3, and their access order, known before
+ * retrieval begins, Sec. 2.1), the destination block table, and the KV
+ * geometry (layers, KV heads, head dim; BF16 in the paper, Sec. 5 setup).
+ *
+ * Layouts (all row-major, contiguous):
+ *   chunk  of n tokens:  [L][2][n][H][D]   K before V, one buffer per chunk
+ *   paged plane p=2l+kv: [num_blocks][B][H][D]   one device buffer per
+ *                        (layer, K/V); the caller passes 2L plane pointers,
+ *                        so split or fused K/V caches both fit.
+ *   request token t of a request lives in slot  block_table[t / B] * B + t % B.
+ *
+ * Ownership: the caller owns every buffer it passes (chunks, planes, tables).
+ * The library owns only small internal buffers (descriptor upload slots, an
+ * error word, a staging ring for the copy-engine variant, probe buffers),
+ * kept per device until kvs_shutdown() or process exit.
+ *
+ * Asynchrony: kvs_retrieve / kvs_store enqueue work on the caller's CUDA
+ * stream and return; every host array they are given is consumed before they
+ * return (it may be freed or reused at once).  Chunk buffers and planes must
+ * stay valid and unmodified until the stream reaches the enqueued work.
+ * The return code reports validation and enqueue status; device-side faults
+ * are reported by kvs_check_errors() or by a KVS_F_VALIDATE call.
+ *
+ * Threading: calls may come from several host threads; the library
+ * serialises its own planning.  The work runs on the device that is current
+ * on the calling thread.
+ */
+#ifndef KVS_H
+#define KVS_H
+
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+/* ---- status codes ------------------------------------------------------ */
+#define KVS_OK               0
+#define KVS_ERR_INVALID_ARG (-1)  /* null pointer, bad geometry, token counts that do not
+                                     tile the matched range, misplaced partial chunk      */
+#define KVS_ERR_BOUNDS      (-2)  /* block table shorter than the range, or a block id
+                                     outside [0, num_blocks)                                */
+#define KVS_ERR_ALIAS       (-3)  /* one physical block named twice by one request, or
+                                     (KVS_F_VALIDATE) shared blocks with differing bytes   */
+#define KVS_ERR_CUDA        (-4)  /* a CUDA runtime call failed; see kvs_last_error()     */
+#define KVS_ERR_TIMEOUT     (-5)  /* a bounded device-side wait expired                    */
+#define KVS_ERR_NOMEM       (-6)  /* an internal buffer could not be allocated            */
+#define KVS_ERR_UNSUPPORTED (-7)  /* a forced variant cannot serve these arguments        */
+
+/* ---- residency of a chunk buffer (the fast-tier stand-in) --------------- */
+#define KVS_SRC_HOST_PINNED 1     /* page-locked host memory mapped into the GPU's address
+                                     space (cudaHostAlloc / cudaHostRegister), reached over
+                                     the host link                                          */
+#define KVS_SRC_DEVICE      2     /* device memory of the current GPU (an HBM staging copy) */
+
+/* ---- flags (bitwise OR) --------------------------------------------------- */
+#define KVS_F_VALIDATE       (1u << 0) /* synchronise the stream after the copy and return
+                                          the device error word; also verify that blocks
+                                          shared by several requests receive equal bytes */
+#define KVS_F_FORCE_HOSTLINK (1u << 1) /* host chunks: SMs load/store host memory directly  */
+#define KVS_F_FORCE_HBMCOPY  (1u << 2) /* host chunks: copy engine to/from an HBM staging
+                                          ring, SMs scatter/gather in HBM                    */
+#define KVS_F_FORCE_LDG      (1u << 3) /* kernel flavour: vector loads/stores by all threads */
+#define KVS_F_FORCE_TMA      (1u << 4) /* kernel flavour: bulk async copies (TMA) staged
+                                          through shared memory; 16-byte aligned data only  */
+#define KVS_F_NO_DEDUP       (1u << 5) /* write shared physical blocks once per request      */
+#define KVS_F_MAX_CTAS(n)    ((((uint32_t)(n)) & 0xFFFFu) << 16) /* cap on CTAs, 0 = auto */
+#define KVS_F_GET_MAX_CTAS(f) (((f) >> 16) & 0xFFFFu)
+
+/* Variant identifiers reported by kvs_query_bw. */
+#define KVS_VARIANT_HOSTLINK 1
+#define KVS_VARIANT_HBMCOPY  2
+#define KVS_KERNEL_LDG       1
+#define KVS_KERNEL_TMA       2
+
+/* KV geometry.  elem_bytes is 2 for BF16 KV (1, 2, 4 and 8 are accepted; elements
+ * are copied as opaque bytes).  chunk_tokens must be a multiple of block_size. */
+typedef struct kvs_geometry {
+    int32_t num_layers;     /* L */
+    int32_t num_kv_heads;   /* H */
+    int32_t head_dim;       /* D */
+    int32_t elem_bytes;     /* e */
+    int32_t block_size;     /* B: tokens per paged block (vLLM block)  */
+    int32_t chunk_tokens;   /* C: tokens per full chunk (LMCache: 256) */
+} kvs_geometry;
+
+/* One chunk buffer, [L][2][num_tokens][H][D].  Every chunk of a request holds
+ * chunk_tokens tokens except the last, which may hold fewer (1..C). */
+typedef struct kvs_chunk {
+    void*   base;           /* host (KVS_SRC_HOST_PINNED) or device (KVS_SRC_DEVICE) address */
+    int32_t num_tokens;
+    int32_t residency;      /* KVS_SRC_* */
+} kvs_chunk;
+
+/* One request's matched range [first_token, first_token + num_tokens) and the
+ * chunks that hold it, in token order.  first_token must be a multiple of
+ * chunk_tokens (a prefix starts at 0).  block_table is a HOST array mapping
+ * logical block k of the request to a physical block id in [0, num_blocks);
+ * it must cover ceil((first_token + num_tokens) / B) blocks. */
+typedef struct kvs_request {
+    int64_t          first_token;
+    int64_t          num_tokens;
+    const kvs_chunk* chunks;
+    int32_t          num_chunks;
+    int32_t          block_table_len;
+    const int32_t*   block_table;
+} kvs_request;
+
+/* The paged KV cache: a HOST array of 2L device pointers ordered
+ * K0, V0, K1, V1, ..., each to a [num_blocks][B][H][D] plane. */
+typedef struct kvs_paged_cache {
+    void* const* kv_planes;
+    int64_t      num_blocks;
+} kvs_paged_cache;
+
+/*
+ * Retrieval (fast tier -> GPU): for every request r, chunk j, layer l, K/V kv,
+ * token i of the chunk, head h and dim d,
+ *     plane[2l+kv][slot(s_j + i)][h][d] = chunk_j[l][kv][i][h][d],
+ * with s_j the first request token of chunk j.  Nothing else is written.
+ * A physical block named by several requests (a shared prefix) must carry the
+ * same KV in each; it is written once, from the request that covers the most
+ * of its tokens (the lowest index among equals), unless KVS_F_NO_DEDUP.
+ * Returns KVS_OK or a KVS_ERR_* code (nothing is enqueued on error).
+ */
+int kvs_retrieve(const kvs_geometry* geom, const kvs_paged_cache* cache,
+                 const kvs_request* requests, int32_t num_requests,
+                 void* cuda_stream, uint32_t flags);
+
+/*
+ * Store-back (GPU -> chunks): the same correspondence read the other way,
+ *     chunk_j[l][kv][i][h][d] = plane[2l+kv][slot(s_j + i)][h][d];
+ * the chunks are the destinations.  The cache is only read.  Destination
+ * chunks must not overlap each other or any plane.
+ */
+int kvs_store(const kvs_geometry* geom, const kvs_paged_cache* cache,
+              const kvs_request* requests, int32_t num_requests,
+              void* cuda_stream, uint32_t flags);
+
+/* Bandwidths measured by kvs_query_bw, in GB/s (1e9 bytes per second). */
+typedef struct kvs_bw_report {
+    double  hbm_copy_gbs;          /* device->device copy kernel, read + write bytes      */
+    double  h2d_copy_engine_gbs;   /* cudaMemcpyAsync pinned host -> device                */
+    double  d2h_copy_engine_gbs;   /* cudaMemcpyAsync device -> pinned host                */
+    double  zero_copy_read_gbs;    /* copy kernel reading pinned host, writing HBM         */
+    double  zero_copy_write_gbs;   /* copy kernel reading HBM, writing pinned host         */
+    double  retrieve_gbs[2];       /* host-chunk retrieval probe: [HOSTLINK, HBMCOPY]      */
+    double  store_gbs[2];          /* host-chunk store probe:     [HOSTLINK, HBMCOPY]      */
+    double  device_kernel_gbs[2];  /* device-chunk retrieval probe, payload bytes: [LDG, TMA] */
+    int32_t chosen_retrieve_host;  /* KVS_VARIANT_* used for host chunks by kvs_retrieve   */
+    int32_t chosen_store_host;     /* KVS_VARIANT_* used for host chunks by kvs_store      */
+    int32_t chosen_kernel_device;  /* KVS_KERNEL_* used for device-resident chunks         */
+    int32_t num_sms;
+    int64_t probe_bytes;           /* bytes moved per probe                                */
+} kvs_bw_report;
+
+/*
+ * Measures the bandwidths above on the current device with probes of
+ * probe_bytes bytes (0 = 1 GiB), synchronously, using cuda_stream, and makes
+ * the measured fastest variants the defaults of later kvs_retrieve / kvs_store
+ * calls on this device.  Allocates (and frees before returning) probe
+ * buffers: 2 * probe_bytes of device memory and probe_bytes of pinned host
+ * memory.  `out` may be NULL.
+ */
+int kvs_query_bw(kvs_bw_report* out, void* cuda_stream, int64_t probe_bytes);
+
+/* Reads the defaults currently in force on this device (after kvs_query_bw,
+ * or the built-in ones) into `out`; bandwidth fields are 0 if never measured. */
+int kvs_get_choice(kvs_bw_report* out);
+
+/*
+ * Synchronises cuda_stream, then reads and clears this device's error word.
+ * Returns KVS_OK, or the first KVS_ERR_* a kernel recorded since the last check.
+ */
+int kvs_check_errors(void* cuda_stream);
+
+/* Message describing the last error on the calling thread ("" if none). */
+const char* kvs_last_error(void);
+
+/* Frees every library-owned buffer on every device (device must be idle). */
+int kvs_shutdown(void);
+
+/*
+ * Self-test of the bounded device-side wait used by the TMA kernel: one CTA
+ * waits on a barrier phase that nothing completes, gives up after limit_ns
+ * (at most 2e9) and records KVS_ERR_TIMEOUT in the error word; the call then
+ * synchronises cuda_stream and returns (and clears) that code.  A correct
+ * build returns KVS_ERR_TIMEOUT and leaves the context usable.
+ */
+int kvs_selftest_wait_timeout(void* cuda_stream, int64_t limit_ns);
+
+/* Number of kernels this library has launched in this process (all devices). */
+int64_t kvs_stat_launches(void);
+
+/* ABI version of this header: major * 10000 + minor * 100 + patch. */
+int kvs_version(void);
+#define KVS_VERSION 10000
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* KVS_H */

@@ -1,0 +1,788 @@
+// kvs_api.cpp -- C ABI, argument validation, planning and variant choice for
+// prefix-KV retrieval / store-back (declared in include/kvs.h).
+//
+// A call is planned on the host: every (request, chunk) pair becomes one
+// Entry, every block of a chunk one physical block id, and the 2L plane
+// pointers one table.  The three arrays go to the device in one upload (a
+// pinned slot copied on the caller's stream), then one kernel per source class
+// moves the bytes:
+//   device-resident chunks  -> LDG or TMA kernel, HBM to HBM;
+//   host-resident chunks    -> HOSTLINK: the LDG kernel loads/stores host memory
+//                              over the host link directly, or
+//                              HBMCOPY: the copy engine moves whole chunks
+//                              through a ring of HBM staging slots and the
+//                              device kernel scatters/gathers from there.
+#include <algorithm>
+#include <chrono>
+#include <cstdarg>
+#include <cstdio>
+#include <cstring>
+#include <mutex>
+#include <string>
+#include <vector>
+
+#include "kvs.h"
+#include "kvs_internal.h"
+
+namespace kvs {
+namespace {
+
+thread_local std::string t_error;
+
+int fail(int code, const char* fmt, ...) {
+    char buf[512];
+    va_list ap;
+    va_start(ap, fmt);
+    vsnprintf(buf, sizeof buf, fmt, ap);
+    va_end(ap);
+    t_error = buf;
+    return code;
+}
+
+#define KVS_CUDA(call)                                                                  \
+    do {                                                                                \
+        cudaError_t e_ = (call);                                                        \
+        if (e_ != cudaSuccess)                                                          \
+            return fail(KVS_ERR_CUDA, "%s failed: %s", #call, cudaGetErrorString(e_));  \
+    } while (0)
+
+constexpr int kUploadSlots = 4;
+constexpr int kRingSlots = 4;
+constexpr uint64_t kRingMinSlotBytes = 64ull << 20;
+
+struct UploadSlot {
+    void*       host = nullptr;   // pinned
+    void*       dev = nullptr;
+    size_t      cap = 0;
+    cudaEvent_t done = nullptr;   // recorded after the last kernel that reads `dev`
+    bool        used = false;
+};
+
+struct DevState {
+    bool         ready = false;
+    int          device = -1;
+    int          sms = 0;
+    int32_t*     err = nullptr;          // device error word
+    int32_t*     err_host = nullptr;     // pinned read-back
+    UploadSlot   up[kUploadSlots];
+    int          next_up = 0;
+    // HBM staging ring of the HBMCOPY variant
+    uint8_t*     ring = nullptr;
+    uint64_t     ring_slot_bytes = 0;
+    cudaStream_t copy_stream = nullptr;
+    cudaEvent_t  ring_filled[kRingSlots] = {};
+    cudaEvent_t  ring_free[kRingSlots] = {};
+    cudaEvent_t  ev_fork = nullptr, ev_join = nullptr;
+    // per-block ownership for de-duplication: stamp[b] == gen -> owner[b] valid
+    std::vector<uint32_t> stamp;
+    std::vector<int64_t>  owner;
+    uint32_t     gen = 0;
+    // defaults (kvs_query_bw may change them)
+    int          retrieve_host = KVS_VARIANT_HOSTLINK;
+    int          store_host = KVS_VARIANT_HOSTLINK;
+    int          kernel_device = KVS_KERNEL_LDG;
+    kvs_bw_report report{};
+};
+
+std::mutex g_mu;
+std::vector<DevState> g_dev;
+int64_t g_launches = 0;
+
+int get_state(DevState** out) {
+    int dev = 0;
+    KVS_CUDA(cudaGetDevice(&dev));
+    if ((int)g_dev.size() <= dev) g_dev.resize(dev + 1);
+    DevState& st = g_dev[dev];
+    if (!st.ready) {
+        st.device = dev;
+        KVS_CUDA(cudaDeviceGetAttribute(&st.sms, cudaDevAttrMultiProcessorCount, dev));
+        KVS_CUDA(cudaMalloc(&st.err, sizeof(int32_t)));
+        KVS_CUDA(cudaMemset(st.err, 0, sizeof(int32_t)));
+        KVS_CUDA(cudaHostAlloc(&st.err_host, sizeof(int32_t), cudaHostAllocDefault));
+        for (auto& s : st.up) KVS_CUDA(cudaEventCreateWithFlags(&s.done, cudaEventDisableTiming));
+        KVS_CUDA(cudaStreamCreateWithFlags(&st.copy_stream, cudaStreamNonBlocking));
+        for (int k = 0; k < kRingSlots; ++k) {
+            KVS_CUDA(cudaEventCreateWithFlags(&st.ring_filled[k], cudaEventDisableTiming));
+            KVS_CUDA(cudaEventCreateWithFlags(&st.ring_free[k], cudaEventDisableTiming));
+        }
+        KVS_CUDA(cudaEventCreateWithFlags(&st.ev_fork, cudaEventDisableTiming));
+        KVS_CUDA(cudaEventCreateWithFlags(&st.ev_join, cudaEventDisableTiming));
+        st.report.num_sms = st.sms;
+        st.report.chosen_retrieve_host = st.retrieve_host;
+        st.report.chosen_store_host = st.store_host;
+        st.report.chosen_kernel_device = st.kernel_device;
+        st.ready = true;
+    }
+    *out = &st;
+    return KVS_OK;
+}
+
+// ---------------------------------------------------------------------------
+// Planning
+// ---------------------------------------------------------------------------
+struct Plan {
+    std::vector<uint64_t> planes;
+    std::vector<Entry>    entries;       // device-resident first, then host-resident
+    std::vector<int32_t>  blocks;        // entries.size() * bpc
+    std::vector<int32_t>  demoted;       // block of a writer dropped by de-duplication, else -1
+    std::vector<int32_t>  blocks_cmp;    // KVS_F_VALIDATE: the demoted writers, compared
+    std::vector<uint64_t> entry_bytes;   // bytes of each entry's chunk buffer
+    uint32_t num_device = 0, num_host = 0;
+    uint32_t bpc = 0;
+    uint64_t row_bytes = 0;
+    uint64_t addr_or = 0;                // OR of all addresses and strides (alignment)
+    bool     any_dedup = false;
+};
+
+bool is_pow2_elem(int e) { return e == 1 || e == 2 || e == 4 || e == 8; }
+
+int validate_geometry(const kvs_geometry* g) {
+    if (!g) return fail(KVS_ERR_INVALID_ARG, "geometry is NULL");
+    if (g->num_layers <= 0 || g->num_kv_heads <= 0 || g->head_dim <= 0)
+        return fail(KVS_ERR_INVALID_ARG, "layers, kv heads and head dim must be positive");
+    if (!is_pow2_elem(g->elem_bytes))
+        return fail(KVS_ERR_INVALID_ARG, "elem_bytes must be 1, 2, 4 or 8 (got %d)", g->elem_bytes);
+    if (g->block_size <= 0 || g->chunk_tokens <= 0 || g->chunk_tokens % g->block_size)
+        return fail(KVS_ERR_INVALID_ARG, "chunk_tokens (%d) must be a positive multiple of block_size (%d)",
+                    g->chunk_tokens, g->block_size);
+    if ((int64_t)g->num_layers * 2 > 65536)
+        return fail(KVS_ERR_INVALID_ARG, "too many layers");
+    return KVS_OK;
+}
+
+// First half of planning: checks every argument and counts entries per class.
+// Touches no CUDA state, so invalid calls fail the same way with or without a GPU.
+int validate_call(const kvs_geometry* g, const kvs_paged_cache* cache,
+                  const kvs_request* reqs, int32_t nreq, Plan& pl) {
+    int rc = validate_geometry(g);
+    if (rc) return rc;
+    if (!cache || !cache->kv_planes) return fail(KVS_ERR_INVALID_ARG, "cache or its plane array is NULL");
+    if (cache->num_blocks <= 0 || cache->num_blocks > INT32_MAX)
+        return fail(KVS_ERR_INVALID_ARG, "num_blocks must be in [1, 2^31)");
+    if (nreq < 0 || (nreq > 0 && !reqs)) return fail(KVS_ERR_INVALID_ARG, "bad request array");
+
+    const int L = g->num_layers, B = g->block_size, C = g->chunk_tokens;
+    const int P = 2 * L;
+    pl.row_bytes = (uint64_t)g->num_kv_heads * g->head_dim * g->elem_bytes;
+    pl.bpc = (uint32_t)((C + B - 1) / B);
+    pl.addr_or = pl.row_bytes;
+    pl.planes.resize(P);
+    for (int p = 0; p < P; ++p) {
+        if (!cache->kv_planes[p]) return fail(KVS_ERR_INVALID_ARG, "plane %d is NULL", p);
+        pl.planes[p] = (uint64_t)cache->kv_planes[p];
+        pl.addr_or |= pl.planes[p];
+    }
+    // Validate requests, count entries per class.
+    for (int32_t r = 0; r < nreq; ++r) {
+        const kvs_request& q = reqs[r];
+        if (q.first_token < 0 || q.first_token % C)
+            return fail(KVS_ERR_INVALID_ARG, "request %d: first_token %lld is not a non-negative multiple of %d",
+                        r, (long long)q.first_token, C);
+        if (q.num_tokens < 0 || q.num_chunks < 0 || (q.num_chunks > 0 && !q.chunks))
+            return fail(KVS_ERR_INVALID_ARG, "request %d: bad token or chunk count", r);
+        if (q.first_token + q.num_tokens > INT32_MAX)
+            return fail(KVS_ERR_INVALID_ARG, "request %d: token range too large", r);
+        int64_t sum = 0;
+        for (int32_t j = 0; j < q.num_chunks; ++j) {
+            const kvs_chunk& c = q.chunks[j];
+            if (!c.base) return fail(KVS_ERR_INVALID_ARG, "request %d chunk %d: base is NULL", r, j);
+            if (c.residency != KVS_SRC_HOST_PINNED && c.residency != KVS_SRC_DEVICE)
+                return fail(KVS_ERR_INVALID_ARG, "request %d chunk %d: unknown residency %d", r, j, c.residency);
+            if (c.num_tokens <= 0 || c.num_tokens > C)
+                return fail(KVS_ERR_INVALID_ARG, "request %d chunk %d: num_tokens %d not in [1, %d]",
+                            r, j, c.num_tokens, C);
+            if (j + 1 < q.num_chunks && c.num_tokens != C)
+                return fail(KVS_ERR_INVALID_ARG, "request %d chunk %d: only the last chunk may be partial", r, j);
+            sum += c.num_tokens;
+            if (c.residency == KVS_SRC_DEVICE) ++pl.num_device; else ++pl.num_host;
+        }
+        if (sum != q.num_tokens)
+            return fail(KVS_ERR_INVALID_ARG, "request %d: chunks hold %lld tokens, num_tokens is %lld",
+                        r, (long long)sum, (long long)q.num_tokens);
+        if (q.num_tokens > 0) {
+            const int64_t need = (q.first_token + q.num_tokens + B - 1) / B;
+            if (!q.block_table) return fail(KVS_ERR_INVALID_ARG, "request %d: block_table is NULL", r);
+            if (q.block_table_len < need)
+                return fail(KVS_ERR_BOUNDS, "request %d: block table has %d entries, %lld needed",
+                            r, q.block_table_len, (long long)need);
+            for (int64_t k = q.first_token / B; k < need; ++k) {
+                const int32_t b = q.block_table[k];
+                if (b < 0 || b >= cache->num_blocks)
+                    return fail(KVS_ERR_BOUNDS, "request %d: block_table[%lld] = %d outside [0, %lld)",
+                                r, (long long)k, b, (long long)cache->num_blocks);
+            }
+        }
+    }
+
+    const uint32_t nent = pl.num_device + pl.num_host;
+    const uint64_t runs = (uint64_t)nent * P * pl.bpc;
+    const uint64_t ppr = ((uint64_t)B * pl.row_bytes + kPieceBytes - 1) / kPieceBytes;
+    if (runs * ppr >= (1ull << 31))
+        return fail(KVS_ERR_INVALID_ARG, "call too large: split it (more than 2^31 pieces)");
+    return KVS_OK;
+}
+
+// Second half: entries, block ids and de-duplication of shared physical blocks.
+int fill_plan(DevState& st, const kvs_geometry* g, const kvs_paged_cache* cache,
+              const kvs_request* reqs, int32_t nreq, bool retrieve, uint32_t flags, Plan& pl) {
+    const int B = g->block_size;
+    const int P = 2 * g->num_layers;
+    const bool validate = flags & KVS_F_VALIDATE;
+    const bool dedup = retrieve && !(flags & KVS_F_NO_DEDUP);
+    const uint32_t nent = pl.num_device + pl.num_host;
+    pl.entries.resize(nent);
+    pl.entry_bytes.resize(nent);
+    pl.blocks.assign((size_t)nent * pl.bpc, -1);
+
+    if (dedup) {
+        if (st.stamp.size() < (size_t)cache->num_blocks) {
+            st.stamp.assign(cache->num_blocks, 0);
+            st.owner.assign(cache->num_blocks, -1);
+            st.gen = 0;
+        }
+        if (++st.gen == 0) {                      // stamp wrap-around
+            std::fill(st.stamp.begin(), st.stamp.end(), 0);
+            st.gen = 1;
+        }
+    }
+
+    uint32_t di = 0, hi = pl.num_device;
+    for (int32_t r = 0; r < nreq; ++r) {
+        const kvs_request& q = reqs[r];
+        int64_t s = q.first_token;
+        for (int32_t j = 0; j < q.num_chunks; ++j) {
+            const kvs_chunk& c = q.chunks[j];
+            const uint32_t e = (c.residency == KVS_SRC_DEVICE) ? di++ : hi++;
+            uint64_t addr = (uint64_t)c.base;
+            if (validate) {
+                cudaPointerAttributes at{};
+                if (cudaPointerGetAttributes(&at, c.base) != cudaSuccess) {
+                    cudaGetLastError();
+                    return fail(KVS_ERR_INVALID_ARG, "request %d chunk %d: unknown pointer", r, j);
+                }
+                if (c.residency == KVS_SRC_DEVICE &&
+                    !(at.type == cudaMemoryTypeDevice || at.type == cudaMemoryTypeManaged))
+                    return fail(KVS_ERR_INVALID_ARG, "request %d chunk %d: not device memory", r, j);
+                if (c.residency == KVS_SRC_HOST_PINNED) {
+                    if (at.type != cudaMemoryTypeHost || !at.devicePointer)
+                        return fail(KVS_ERR_INVALID_ARG, "request %d chunk %d: not mapped page-locked host memory", r, j);
+                    addr = (uint64_t)at.devicePointer;
+                }
+            }
+            pl.entries[e].chunk = addr;
+            pl.entries[e].n_tok = c.num_tokens;
+            pl.entries[e].blk_off = (int32_t)((uint64_t)e * pl.bpc);
+            pl.entry_bytes[e] = (uint64_t)P * c.num_tokens * pl.row_bytes;
+            pl.addr_or |= addr;
+            for (int32_t i = 0; i * B < c.num_tokens; ++i) {
+                const int64_t t = s + (int64_t)i * B;
+                const int32_t blk = q.block_table[t / B];
+                const int32_t ntok = std::min<int32_t>(B, c.num_tokens - i * B);
+                const int64_t me = ((int64_t)r << 32) | ((int64_t)e * pl.bpc + i);
+                if (dedup) {
+                    if (st.stamp[blk] == st.gen) {
+                        const int64_t prev = st.owner[blk];
+                        const int32_t prev_req = (int32_t)(prev >> 32);
+                        const int64_t prev_slot = prev & 0xffffffffll;
+                        if (prev_req == r)
+                            return fail(KVS_ERR_ALIAS, "request %d names physical block %d twice", r, blk);
+                        if (!pl.any_dedup) pl.demoted.assign(pl.blocks.size(), -1);
+                        pl.any_dedup = true;
+                        // keep the writer covering more tokens (earlier request on ties)
+                        const uint32_t pe = (uint32_t)(prev_slot / pl.bpc);
+                        const int32_t pi = (int32_t)(prev_slot % pl.bpc);
+                        const int32_t prev_ntok = std::min<int32_t>(B, pl.entries[pe].n_tok - pi * B);
+                        const int64_t my_slot = (int64_t)e * pl.bpc + i;
+                        if (ntok > prev_ntok) {
+                            pl.blocks[prev_slot] = -1;
+                            pl.demoted[prev_slot] = blk;
+                            pl.blocks[my_slot] = blk;
+                            st.owner[blk] = me;
+                        } else {
+                            pl.demoted[my_slot] = blk;
+                        }
+                        continue;
+                    }
+                    st.stamp[blk] = st.gen;
+                    st.owner[blk] = me;
+                }
+                pl.blocks[(uint64_t)e * pl.bpc + i] = blk;
+            }
+            s += c.num_tokens;
+        }
+    }
+    // With KVS_F_VALIDATE the demoted writers are compared against what the
+    // kept writer put into the block.
+    if (pl.any_dedup && validate) pl.blocks_cmp = pl.demoted;
+    return KVS_OK;
+}
+
+int vec_bytes_for(uint64_t addr_or) {
+    int v = 16;
+    while (v > 1 && (addr_or & (uint64_t)(v - 1))) v >>= 1;
+    return v;
+}
+
+// Copies the plan's tables into an upload slot and onto the device (caller stream).
+struct Uploaded {
+    const Entry*    entries;
+    const int32_t*  blocks;
+    const int32_t*  blocks_cmp;
+    const uint64_t* planes;
+    UploadSlot*     slot;
+};
+
+size_t align_up(size_t x, size_t a) { return (x + a - 1) / a * a; }
+
+int upload(DevState& st, const Plan& pl, cudaStream_t s, Uploaded& u) {
+    const size_t b_pl = align_up(pl.planes.size() * 8, 256);
+    const size_t b_en = align_up(pl.entries.size() * sizeof(Entry), 256);
+    const size_t b_bl = align_up(pl.blocks.size() * 4, 256);
+    const size_t b_bc = align_up(pl.blocks_cmp.size() * 4, 256);
+    const size_t need = b_pl + b_en + b_bl + b_bc;
+    UploadSlot& sl = st.up[st.next_up];
+    st.next_up = (st.next_up + 1) % kUploadSlots;
+    if (sl.used) KVS_CUDA(cudaEventSynchronize(sl.done));
+    if (sl.cap < need) {
+        if (sl.host) { cudaFreeHost(sl.host); sl.host = nullptr; }
+        if (sl.dev) { cudaFree(sl.dev); sl.dev = nullptr; }
+        const size_t cap = std::max<size_t>(align_up(need * 2, 1 << 16), 1 << 16);
+        if (cudaHostAlloc(&sl.host, cap, cudaHostAllocDefault) != cudaSuccess ||
+            cudaMalloc(&sl.dev, cap) != cudaSuccess) {
+            cudaGetLastError();
+            sl.cap = 0;
+            return fail(KVS_ERR_NOMEM, "cannot allocate a %zu-byte descriptor slot", cap);
+        }
+        sl.cap = cap;
+    }
+    uint8_t* h = (uint8_t*)sl.host;
+    memcpy(h, pl.planes.data(), pl.planes.size() * 8);
+    memcpy(h + b_pl, pl.entries.data(), pl.entries.size() * sizeof(Entry));
+    memcpy(h + b_pl + b_en, pl.blocks.data(), pl.blocks.size() * 4);
+    if (b_bc) memcpy(h + b_pl + b_en + b_bl, pl.blocks_cmp.data(), pl.blocks_cmp.size() * 4);
+    KVS_CUDA(cudaMemcpyAsync(sl.dev, sl.host, need, cudaMemcpyHostToDevice, s));
+    uint8_t* d = (uint8_t*)sl.dev;
+    u.planes = (const uint64_t*)d;
+    u.entries = (const Entry*)(d + b_pl);
+    u.blocks = (const int32_t*)(d + b_pl + b_en);
+    u.blocks_cmp = b_bc ? (const int32_t*)(d + b_pl + b_en + b_bl) : nullptr;
+    u.slot = &sl;
+    return KVS_OK;
+}
+
+Job make_job(DevState& st, const kvs_geometry* g, const kvs_paged_cache* cache, const Plan& pl,
+             const Uploaded& u, uint32_t first_entry, uint32_t num_entries, Mode mode) {
+    Job j{};
+    j.entries = u.entries + first_entry;
+    j.blocks = u.blocks;
+    j.planes = u.planes;
+    j.err = st.err;
+    j.row_bytes = pl.row_bytes;
+    j.num_blocks = cache->num_blocks;
+    j.num_entries = num_entries;
+    j.num_planes = (uint32_t)pl.planes.size();
+    j.blocks_per_chunk = pl.bpc;
+    j.piece_bytes = kPieceBytes;
+    j.block_size = (uint32_t)g->block_size;
+    const uint64_t run_max = (uint64_t)g->block_size * pl.row_bytes;
+    j.pieces_per_run = (uint32_t)((run_max + kPieceBytes - 1) / kPieceBytes);
+    j.num_pieces = (uint64_t)num_entries * j.num_planes * j.blocks_per_chunk * j.pieces_per_run;
+    j.mode = mode;
+    return j;
+}
+
+int launch_kernel(const Job& j, int flavour, int vec, int grid, cudaStream_t s) {
+    if (j.num_pieces == 0) return KVS_OK;
+    cudaError_t e = (flavour == KVS_KERNEL_TMA) ? launch_tma(j, grid, s) : launch_ldg(j, vec, grid, s);
+    if (e != cudaSuccess) return fail(KVS_ERR_CUDA, "kernel launch failed: %s", cudaGetErrorString(e));
+    ++g_launches;
+    return KVS_OK;
+}
+
+int ensure_ring(DevState& st, uint64_t max_entry_bytes, cudaStream_t s) {
+    const uint64_t want = std::max<uint64_t>(kRingMinSlotBytes, align_up(max_entry_bytes, 1 << 20));
+    if (st.ring && st.ring_slot_bytes >= want) return KVS_OK;
+    if (st.ring) {
+        KVS_CUDA(cudaStreamSynchronize(s));
+        KVS_CUDA(cudaStreamSynchronize(st.copy_stream));
+        KVS_CUDA(cudaFree(st.ring));
+        st.ring = nullptr;
+    }
+    if (cudaMalloc(&st.ring, want * kRingSlots) != cudaSuccess) {
+        cudaGetLastError();
+        st.ring_slot_bytes = 0;
+        return fail(KVS_ERR_NOMEM, "cannot allocate the %llu-byte HBM staging ring",
+                    (unsigned long long)(want * kRingSlots));
+    }
+    st.ring_slot_bytes = want;
+    return KVS_OK;
+}
+
+// Host chunks through the copy engine and the HBM ring.  Batches of whole
+// chunks fill one ring slot each; the copy stream and the caller's stream
+// hand slots back and forth with events.
+int run_hbmcopy(DevState& st, const kvs_geometry* g, const kvs_paged_cache* cache, Plan& pl,
+                const Uploaded& u, Mode mode, int flavour, int grid, cudaStream_t s,
+                const std::vector<const void*>& host_addr) {
+    uint64_t max_bytes = 0;
+    for (uint32_t e = pl.num_device; e < pl.entries.size(); ++e) max_bytes = std::max(max_bytes, pl.entry_bytes[e]);
+    int rc = ensure_ring(st, max_bytes, s);
+    if (rc) return rc;
+    // Entries in the device copy of the table still point at host memory; the
+    // ring kernels use a second upload whose chunk addresses point into slots.
+    Plan ring_plan = pl;
+    std::vector<uint32_t> batch_first, batch_slot;
+    uint64_t used = st.ring_slot_bytes;    // force a new batch at the first entry
+    int slot = -1, nb = 0;
+    for (uint32_t e = pl.num_device; e < pl.entries.size(); ++e) {
+        const uint64_t b = align_up(pl.entry_bytes[e], 256);
+        if (used + b > st.ring_slot_bytes) {
+            slot = (slot + 1) % kRingSlots;
+            batch_first.push_back(e);
+            batch_slot.push_back((uint32_t)slot);
+            used = 0;
+            ++nb;
+        }
+        ring_plan.entries[e].chunk = (uint64_t)(st.ring + (uint64_t)slot * st.ring_slot_bytes + used);
+        ring_plan.addr_or |= ring_plan.entries[e].chunk;
+        used += b;
+    }
+    batch_first.push_back((uint32_t)pl.entries.size());
+    Uploaded ru;
+    rc = upload(st, ring_plan, s, ru);
+    if (rc) return rc;
+    const int vec = vec_bytes_for(ring_plan.addr_or);
+    if (flavour == KVS_KERNEL_TMA && vec != 16) flavour = KVS_KERNEL_LDG;
+
+    KVS_CUDA(cudaEventRecord(st.ev_fork, s));
+    KVS_CUDA(cudaStreamWaitEvent(st.copy_stream, st.ev_fork, 0));
+    for (int b = 0; b < nb; ++b) {
+        const uint32_t e0 = batch_first[b], e1 = batch_first[b + 1];
+        const int k = (int)batch_slot[b];
+        Job j = make_job(st, g, cache, ring_plan, ru, e0, e1 - e0, mode);
+        if (mode == MODE_RETRIEVE) {
+            KVS_CUDA(cudaStreamWaitEvent(st.copy_stream, st.ring_free[k], 0));
+            for (uint32_t e = e0; e < e1; ++e)
+                KVS_CUDA(cudaMemcpyAsync((void*)ring_plan.entries[e].chunk, host_addr[e - pl.num_device],
+                                         pl.entry_bytes[e], cudaMemcpyHostToDevice, st.copy_stream));
+            KVS_CUDA(cudaEventRecord(st.ring_filled[k], st.copy_stream));
+            KVS_CUDA(cudaStreamWaitEvent(s, st.ring_filled[k], 0));
+            rc = launch_kernel(j, flavour, vec, grid, s);
+            if (rc) return rc;
+            KVS_CUDA(cudaEventRecord(st.ring_free[k], s));
+        } else {
+            KVS_CUDA(cudaStreamWaitEvent(s, st.ring_free[k], 0));
+            rc = launch_kernel(j, flavour, vec, grid, s);
+            if (rc) return rc;
+            KVS_CUDA(cudaEventRecord(st.ring_filled[k], s));
+            KVS_CUDA(cudaStreamWaitEvent(st.copy_stream, st.ring_filled[k], 0));
+            for (uint32_t e = e0; e < e1; ++e)
+                KVS_CUDA(cudaMemcpyAsync((void*)host_addr[e - pl.num_device], (const void*)ring_plan.entries[e].chunk,
+                                         pl.entry_bytes[e], cudaMemcpyDeviceToHost, st.copy_stream));
+            KVS_CUDA(cudaEventRecord(st.ring_free[k], st.copy_stream));
+        }
+    }
+    KVS_CUDA(cudaEventRecord(st.ev_join, st.copy_stream));
+    KVS_CUDA(cudaStreamWaitEvent(s, st.ev_join, 0));
+    KVS_CUDA(cudaEventRecord(ru.slot->done, s));
+    ru.slot->used = true;
+    return KVS_OK;
+}
+
+int read_error_word(DevState& st, cudaStream_t s) {
+    KVS_CUDA(cudaMemcpyAsync(st.err_host, st.err, sizeof(int32_t), cudaMemcpyDeviceToHost, s));
+    KVS_CUDA(cudaStreamSynchronize(s));
+    const int32_t code = *st.err_host;
+    if (code != 0) {
+        KVS_CUDA(cudaMemsetAsync(st.err, 0, sizeof(int32_t), s));
+        KVS_CUDA(cudaStreamSynchronize(s));
+        return fail(code, "device reported error %d", code);
+    }
+    return KVS_OK;
+}
+
+int copy_call(const kvs_geometry* g, const kvs_paged_cache* cache, const kvs_request* reqs,
+              int32_t nreq, void* stream, uint32_t flags, bool retrieve) {
+    const bool f_host = flags & KVS_F_FORCE_HOSTLINK, f_hbm = flags & KVS_F_FORCE_HBMCOPY;
+    const bool f_ldg = flags & KVS_F_FORCE_LDG, f_tma = flags & KVS_F_FORCE_TMA;
+    if ((f_host && f_hbm) || (f_ldg && f_tma))
+        return fail(KVS_ERR_INVALID_ARG, "conflicting FORCE flags");
+    Plan pl;
+    int rc = validate_call(g, cache, reqs, nreq, pl);
+    if (rc) return rc;
+    if (pl.num_device + pl.num_host == 0) return KVS_OK;
+    DevState* stp = nullptr;
+    rc = get_state(&stp);
+    if (rc) return rc;
+    DevState& st = *stp;
+    cudaStream_t s = (cudaStream_t)stream;
+    rc = fill_plan(st, g, cache, reqs, nreq, retrieve, flags, pl);
+    if (rc) return rc;
+    const int grid = (int)KVS_F_GET_MAX_CTAS(flags);
+    const int vec = vec_bytes_for(pl.addr_or);
+    int flavour = f_tma ? KVS_KERNEL_TMA : f_ldg ? KVS_KERNEL_LDG : st.kernel_device;
+    if (flavour == KVS_KERNEL_TMA && vec != 16) {
+        if (f_tma) return fail(KVS_ERR_UNSUPPORTED, "TMA needs 16-byte aligned chunks, planes and rows");
+        flavour = KVS_KERNEL_LDG;
+    }
+    const int host_variant = f_host ? KVS_VARIANT_HOSTLINK : f_hbm ? KVS_VARIANT_HBMCOPY
+                                                                    : (retrieve ? st.retrieve_host : st.store_host);
+    const Mode mode = retrieve ? MODE_RETRIEVE : MODE_STORE;
+
+    Uploaded u;
+    rc = upload(st, pl, s, u);
+    if (rc) return rc;
+    if (pl.num_device) {
+        rc = launch_kernel(make_job(st, g, cache, pl, u, 0, pl.num_device, mode), flavour, vec, grid, s);
+        if (rc) return rc;
+    }
+    if (pl.num_host) {
+        if (host_variant == KVS_VARIANT_HBMCOPY) {
+            std::vector<const void*> host_addr(pl.num_host);
+            for (uint32_t e = pl.num_device; e < pl.entries.size(); ++e)
+                host_addr[e - pl.num_device] = (const void*)pl.entries[e].chunk;
+            rc = run_hbmcopy(st, g, cache, pl, u, mode, flavour, grid, s, host_addr);
+        } else {
+            rc = launch_kernel(make_job(st, g, cache, pl, u, pl.num_device, pl.num_host, mode),
+                               KVS_KERNEL_LDG, vec, grid, s);
+        }
+        if (rc) return rc;
+    }
+    if (!pl.blocks_cmp.empty()) {
+        Job j = make_job(st, g, cache, pl, u, 0, (uint32_t)pl.entries.size(), MODE_COMPARE);
+        j.blocks = u.blocks_cmp;
+        rc = launch_kernel(j, KVS_KERNEL_LDG, vec, grid, s);
+        if (rc) return rc;
+    }
+    KVS_CUDA(cudaEventRecord(u.slot->done, s));
+    u.slot->used = true;
+    if (flags & KVS_F_VALIDATE) return read_error_word(st, s);
+    return KVS_OK;
+}
+
+// ---------------------------------------------------------------------------
+// Bandwidth probes
+// ---------------------------------------------------------------------------
+template <class F>
+int time_best(cudaStream_t s, int reps, double* best_ms, F&& body) {
+    cudaEvent_t a, b;
+    KVS_CUDA(cudaEventCreate(&a));
+    KVS_CUDA(cudaEventCreate(&b));
+    *best_ms = 1e30;
+    for (int r = 0; r < reps + 1; ++r) {                 // first run warms up
+        KVS_CUDA(cudaEventRecord(a, s));
+        int rc = body();
+        if (rc) { cudaEventDestroy(a); cudaEventDestroy(b); return rc; }
+        KVS_CUDA(cudaEventRecord(b, s));
+        KVS_CUDA(cudaEventSynchronize(b));
+        float ms = 0;
+        KVS_CUDA(cudaEventElapsedTime(&ms, a, b));
+        if (r > 0) *best_ms = std::min(*best_ms, (double)ms);
+    }
+    cudaEventDestroy(a);
+    cudaEventDestroy(b);
+    return KVS_OK;
+}
+
+int query_bw(DevState& st, kvs_bw_report* out, cudaStream_t s, int64_t probe_bytes) {
+    if (probe_bytes <= 0) probe_bytes = 1ll << 30;
+    probe_bytes = std::max<int64_t>(probe_bytes & ~((int64_t)(8 << 20) - 1), 16 << 20);
+    const uint64_t n = (uint64_t)probe_bytes;
+    kvs_bw_report rep{};
+    rep.num_sms = st.sms;
+    rep.probe_bytes = probe_bytes;
+    uint8_t *d0 = nullptr, *d1 = nullptr, *h = nullptr;
+    auto cleanup = [&]() {
+        if (d0) cudaFree(d0);
+        if (d1) cudaFree(d1);
+        if (h) cudaFreeHost(h);
+    };
+    if (cudaMalloc(&d0, n) != cudaSuccess || cudaMalloc(&d1, n) != cudaSuccess ||
+        cudaHostAlloc(&h, n, cudaHostAllocDefault) != cudaSuccess) {
+        cudaGetLastError();
+        cleanup();
+        return fail(KVS_ERR_NOMEM, "cannot allocate %lld-byte probe buffers", (long long)probe_bytes);
+    }
+    int rc = KVS_OK;
+    double ms = 0;
+    const int reps = 5;
+#define PROBE(field, scale, body)                                               \
+    do {                                                                        \
+        rc = time_best(s, reps, &ms, [&]() -> int { body; return KVS_OK; });    \
+        if (rc) { cleanup(); return rc; }                                       \
+        rep.field = (scale) * (double)n / (ms * 1e6);                           \
+    } while (0)
+    KVS_CUDA(cudaMemsetAsync(d0, 1, n, s));
+    memset(h, 2, n);
+    PROBE(hbm_copy_gbs, 2.0, KVS_CUDA(launch_flat_copy(d1, d0, n, 0, s)); ++g_launches);
+    PROBE(h2d_copy_engine_gbs, 1.0, KVS_CUDA(cudaMemcpyAsync(d0, h, n, cudaMemcpyHostToDevice, s)));
+    PROBE(d2h_copy_engine_gbs, 1.0, KVS_CUDA(cudaMemcpyAsync(h, d0, n, cudaMemcpyDeviceToHost, s)));
+    PROBE(zero_copy_read_gbs, 1.0, KVS_CUDA(launch_flat_copy(d0, h, n, 0, s)); ++g_launches);
+    PROBE(zero_copy_write_gbs, 1.0, KVS_CUDA(launch_flat_copy(h, d0, n, 0, s)); ++g_launches);
+
+    // Scatter / gather probes on an 8B-like geometry: 8 layers, 8 KV heads,
+    // head_dim 128, bf16, B = 16, C = 256 (8 MiB chunks), random block table.
+    kvs_geometry g{8, 8, 128, 2, 16, 256};
+    const uint64_t chunk_bytes = 2ull * g.num_layers * g.chunk_tokens * g.num_kv_heads * g.head_dim * g.elem_bytes;
+    const int nchunks = (int)(n / chunk_bytes);
+    const int64_t tokens = (int64_t)nchunks * g.chunk_tokens;
+    const int64_t nblocks = tokens / g.block_size;
+    const uint64_t plane_bytes = (uint64_t)nblocks * g.block_size * g.num_kv_heads * g.head_dim * g.elem_bytes;
+    std::vector<void*> planes(2 * g.num_layers);
+    for (int p = 0; p < 2 * g.num_layers; ++p) planes[p] = d1 + (uint64_t)p * plane_bytes;
+    std::vector<int32_t> table(nblocks);
+    for (int64_t k = 0; k < nblocks; ++k) table[k] = (int32_t)k;
+    uint64_t x = 0x9E3779B97F4A7C15ull;                          // fixed shuffle (xorshift)
+    for (int64_t k = nblocks - 1; k > 0; --k) {
+        x ^= x << 13; x ^= x >> 7; x ^= x << 17;
+        std::swap(table[k], table[(int64_t)(x % (uint64_t)(k + 1))]);
+    }
+    kvs_paged_cache cache{planes.data(), nblocks};
+    std::vector<kvs_chunk> hc(nchunks), dc(nchunks);
+    for (int c = 0; c < nchunks; ++c) {
+        hc[c] = {h + (uint64_t)c * chunk_bytes, g.chunk_tokens, KVS_SRC_HOST_PINNED};
+        dc[c] = {d0 + (uint64_t)c * chunk_bytes, g.chunk_tokens, KVS_SRC_DEVICE};
+    }
+    kvs_request rh{0, tokens, hc.data(), nchunks, (int32_t)nblocks, table.data()};
+    kvs_request rd{0, tokens, dc.data(), nchunks, (int32_t)nblocks, table.data()};
+    const uint64_t moved = (uint64_t)tokens * chunk_bytes / g.chunk_tokens;
+    auto probe_call = [&](const kvs_request* r, bool retrieve, uint32_t fl, double* field) -> int {
+        double best = 0;
+        int rc2 = time_best(s, reps, &best, [&]() -> int {
+            return copy_call(&g, &cache, r, 1, (void*)s, fl, retrieve);
+        });
+        if (rc2) return rc2;
+        *field = (double)moved / (best * 1e6);
+        return KVS_OK;
+    };
+    if ((rc = probe_call(&rh, true, KVS_F_FORCE_HOSTLINK, &rep.retrieve_gbs[0])) ||
+        (rc = probe_call(&rh, true, KVS_F_FORCE_HBMCOPY, &rep.retrieve_gbs[1])) ||
+        (rc = probe_call(&rh, false, KVS_F_FORCE_HOSTLINK, &rep.store_gbs[0])) ||
+        (rc = probe_call(&rh, false, KVS_F_FORCE_HBMCOPY, &rep.store_gbs[1])) ||
+        (rc = probe_call(&rd, true, KVS_F_FORCE_LDG, &rep.device_kernel_gbs[0])) ||
+        (rc = probe_call(&rd, true, KVS_F_FORCE_TMA, &rep.device_kernel_gbs[1]))) {
+        cleanup();
+        return rc;
+    }
+#undef PROBE
+    KVS_CUDA(cudaStreamSynchronize(s));
+    cleanup();
+    st.retrieve_host = rep.retrieve_gbs[1] > rep.retrieve_gbs[0] ? KVS_VARIANT_HBMCOPY : KVS_VARIANT_HOSTLINK;
+    st.store_host = rep.store_gbs[1] > rep.store_gbs[0] ? KVS_VARIANT_HBMCOPY : KVS_VARIANT_HOSTLINK;
+    st.kernel_device = rep.device_kernel_gbs[1] > rep.device_kernel_gbs[0] ? KVS_KERNEL_TMA : KVS_KERNEL_LDG;
+    rep.chosen_retrieve_host = st.retrieve_host;
+    rep.chosen_store_host = st.store_host;
+    rep.chosen_kernel_device = st.kernel_device;
+    st.report = rep;
+    if (out) *out = rep;
+    return KVS_OK;
+}
+
+}  // namespace
+}  // namespace kvs
+
+using namespace kvs;
+
+extern "C" {
+
+int kvs_retrieve(const kvs_geometry* geom, const kvs_paged_cache* cache, const kvs_request* requests,
+                 int32_t num_requests, void* cuda_stream, uint32_t flags) {
+    std::lock_guard<std::mutex> lk(g_mu);
+    t_error.clear();
+    return copy_call(geom, cache, requests, num_requests, cuda_stream, flags, true);
+}
+
+int kvs_store(const kvs_geometry* geom, const kvs_paged_cache* cache, const kvs_request* requests,
+              int32_t num_requests, void* cuda_stream, uint32_t flags) {
+    std::lock_guard<std::mutex> lk(g_mu);
+    t_error.clear();
+    return copy_call(geom, cache, requests, num_requests, cuda_stream, flags, false);
+}
+
+int kvs_query_bw(kvs_bw_report* out, void* cuda_stream, int64_t probe_bytes) {
+    std::lock_guard<std::mutex> lk(g_mu);
+    t_error.clear();
+    DevState* st = nullptr;
+    int rc = get_state(&st);
+    if (rc) return rc;
+    return query_bw(*st, out, (cudaStream_t)cuda_stream, probe_bytes);
+}
+
+int kvs_get_choice(kvs_bw_report* out) {
+    std::lock_guard<std::mutex> lk(g_mu);
+    t_error.clear();
+    if (!out) return fail(KVS_ERR_INVALID_ARG, "out is NULL");
+    DevState* st = nullptr;
+    int rc = get_state(&st);
+    if (rc) return rc;
+    *out = st->report;
+    out->chosen_retrieve_host = st->retrieve_host;
+    out->chosen_store_host = st->store_host;
+    out->chosen_kernel_device = st->kernel_device;
+    out->num_sms = st->sms;
+    return KVS_OK;
+}
+
+int kvs_check_errors(void* cuda_stream) {
+    std::lock_guard<std::mutex> lk(g_mu);
+    t_error.clear();
+    DevState* st = nullptr;
+    int rc = get_state(&st);
+    if (rc) return rc;
+    return read_error_word(*st, (cudaStream_t)cuda_stream);
+}
+
+const char* kvs_last_error(void) { return t_error.c_str(); }
+
+int kvs_shutdown(void) {
+    std::lock_guard<std::mutex> lk(g_mu);
+    int prev = 0;
+    cudaGetDevice(&prev);
+    for (auto& st : g_dev) {
+        if (!st.ready) continue;
+        cudaSetDevice(st.device);
+        cudaDeviceSynchronize();
+        for (auto& sl : st.up) {
+            if (sl.host) cudaFreeHost(sl.host);
+            if (sl.dev) cudaFree(sl.dev);
+            if (sl.done) cudaEventDestroy(sl.done);
+        }
+        for (int k = 0; k < kRingSlots; ++k) {
+            cudaEventDestroy(st.ring_filled[k]);
+            cudaEventDestroy(st.ring_free[k]);
+        }
+        cudaEventDestroy(st.ev_fork);
+        cudaEventDestroy(st.ev_join);
+        if (st.ring) cudaFree(st.ring);
+        if (st.copy_stream) cudaStreamDestroy(st.copy_stream);
+        if (st.err) cudaFree(st.err);
+        if (st.err_host) cudaFreeHost(st.err_host);
+        st = DevState{};
+    }
+    g_dev.clear();
+    cudaSetDevice(prev);
+    return KVS_OK;
+}
+
+int kvs_version(void) { return KVS_VERSION; }
+
+int64_t kvs_stat_launches(void) {
+    std::lock_guard<std::mutex> lk(g_mu);
+    return g_launches;
+}
+
+int kvs_selftest_wait_timeout(void* cuda_stream, int64_t limit_ns) {
+    std::lock_guard<std::mutex> lk(g_mu);
+    t_error.clear();
+    if (limit_ns <= 0 || limit_ns > 2000000000ll)
+        return fail(KVS_ERR_INVALID_ARG, "limit_ns must be in (0, 2e9]");
+    DevState* st = nullptr;
+    int rc = get_state(&st);
+    if (rc) return rc;
+    cudaStream_t s = (cudaStream_t)cuda_stream;
+    KVS_CUDA(launch_stall(st->err, (uint64_t)limit_ns, s));
+    ++g_launches;
+    return read_error_word(*st, s);
+}
+
+}  // extern "C"

@@ -1,0 +1,60 @@
+// kvs_internal.h -- descriptors shared by the planner (kvs_api.cpp) and the
+// copy kernels (kvs_kernels.cu).  Not part of the public ABI.
+#pragma once
+
+#include <cstdint>
+#include <cuda_runtime.h>
+
+namespace kvs {
+
+// One (request, chunk) pair of a call.  The chunk buffer is [L][2][n_tok][H][D].
+struct Entry {
+    uint64_t chunk;     // device-visible address of the chunk buffer
+    int32_t  n_tok;     // tokens held by the chunk (its token stride)
+    int32_t  blk_off;   // index of the chunk's first block in Job::blocks
+};
+static_assert(sizeof(Entry) == 16, "Entry is uploaded as raw bytes");
+
+enum Mode : int32_t {
+    MODE_RETRIEVE = 0,  // chunk -> plane
+    MODE_STORE    = 1,  // plane -> chunk
+    MODE_COMPARE  = 2,  // flag KVS_ERR_ALIAS where chunk bytes differ from plane bytes
+};
+
+// Work of one launch.  A "run" is the contiguous copy of one (entry, plane p,
+// block i of the chunk): up to B token rows, B*R bytes, contiguous on both
+// sides.  Runs are cut into "pieces" of at most piece_bytes for the kernels.
+// Run index g = (entry * num_planes + p) * blocks_per_chunk + i.
+struct Job {
+    const Entry*    entries;
+    const int32_t*  blocks;          // physical block of (entry, i); < 0 means "skip"
+    const uint64_t* planes;          // 2L plane base addresses
+    int32_t*        err;             // device error word (first error wins)
+    uint64_t        row_bytes;       // R = H * D * e
+    uint64_t        num_pieces;      // num_entries * num_planes * blocks_per_chunk * pieces_per_run
+    int64_t         num_blocks;      // NB, for the device-side bounds check
+    uint32_t        num_entries;
+    uint32_t        num_planes;
+    uint32_t        blocks_per_chunk;
+    uint32_t        pieces_per_run;
+    uint32_t        piece_bytes;     // multiple of 16
+    uint32_t        block_size;      // B
+    int32_t         mode;            // Mode
+};
+
+// Piece size used by both kernel flavours.
+constexpr uint32_t kPieceBytes = 32768;
+
+// Launchers (kvs_kernels.cu).  `grid` <= 0 means "fill the GPU".
+cudaError_t launch_ldg(const Job& job, int vec_bytes, int grid, cudaStream_t s);
+cudaError_t launch_tma(const Job& job, int grid, cudaStream_t s);
+// Contiguous copy of `bytes` (multiple of 16, 16-byte aligned) for bandwidth probes.
+cudaError_t launch_flat_copy(void* dst, const void* src, uint64_t bytes, int grid, cudaStream_t s);
+// One CTA waits (bounded by limit_ns) on an mbarrier phase that nothing
+// completes, then records KVS_ERR_TIMEOUT: exercises the bounded-wait path.
+cudaError_t launch_stall(int32_t* err, uint64_t limit_ns, cudaStream_t s);
+// CTAs per SM the flavour runs with (occupancy); used to size persistent grids.
+int ldg_ctas_per_sm();
+int tma_ctas_per_sm();
+
+}  // namespace kvs

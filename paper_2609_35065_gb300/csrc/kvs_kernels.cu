@@ -1,0 +1,430 @@
+// kvs_kernels.cu -- copy kernels for prefix-KV retrieval / store-back on sm_103a.
+//
+// The work is pure data movement (TempoKV reuses the runtime's transfer path
+// into the paged cache, Sec. 4): every run is one contiguous B*R-byte copy
+// between a chunk buffer [L][2][n][H][D] and one paged block of one
+// (layer, K/V) plane [NB][B][H][D].  Two flavours:
+//
+//  * LDG: all threads of a 256-thread CTA move one 32 KiB piece with
+//    16-byte vector loads (non-coherent, no L1 allocation) issued ahead of
+//    16-byte streaming stores; persistent grid, grid-stride over pieces.
+//    Works for device and mapped-host sources and destinations.
+//  * TMA: one thread per CTA drives a ring of shared-memory stages with 1-D
+//    bulk async copies (cp.async.bulk global->shared completing on an
+//    mbarrier, then shared->global bulk stores); every wait is bounded by the
+//    global timer and reports KVS_ERR_TIMEOUT instead of hanging.
+#include <cstdint>
+
+#include "kvs.h"
+#include "kvs_internal.h"
+
+namespace kvs {
+namespace {
+
+// ---------------------------------------------------------------------------
+// Division by a launch-invariant divisor d, for dividends below 2^31: with
+// p = 31 + ceil(log2 d) and m = ceil(2^p / d), floor(n / d) = (n * m) >> p
+// (round-up reciprocal method; the error term n*(m*d - 2^p)/(d*2^p) stays
+// below 1/d).  m < 2^32 for every d >= 1.
+// ---------------------------------------------------------------------------
+struct FastDiv {
+    uint32_t d, m, p;
+};
+
+FastDiv make_fastdiv(uint32_t d) {
+    uint32_t l = 0;
+    while ((1ull << l) < d) ++l;
+    FastDiv f;
+    f.d = d;
+    f.p = 31 + l;
+    f.m = (uint32_t)(((1ull << f.p) + d - 1) / d);
+    return f;
+}
+
+__device__ __forceinline__ uint32_t fdiv(uint32_t n, const FastDiv& f) {
+    return (uint32_t)(((uint64_t)n * f.m) >> f.p);
+}
+
+struct Decoder {
+    Job job;
+    FastDiv ppr, bpc, planes;
+};
+
+struct Piece {
+    uint64_t chunk_addr;
+    uint64_t plane_addr;
+    uint32_t len;
+};
+
+// Piece q -> addresses.  Returns false for pieces with nothing to move
+// (past the end of a short chunk, a skipped block, a bounds violation).
+__device__ __forceinline__ bool decode_piece(const Decoder& dc, uint32_t q, Piece& pc) {
+    const Job& j = dc.job;
+    const uint32_t g = fdiv(q, dc.ppr);
+    const uint32_t k = q - g * dc.ppr.d;
+    const uint32_t ep = fdiv(g, dc.bpc);
+    const uint32_t i = g - ep * dc.bpc.d;
+    const uint32_t e = fdiv(ep, dc.planes);
+    const uint32_t p = ep - e * dc.planes.d;
+    const Entry en = j.entries[e];
+    const int64_t first = (int64_t)i * j.block_size;
+    const int64_t ntok = min((int64_t)j.block_size, (int64_t)en.n_tok - first);
+    if (ntok <= 0) return false;
+    const int32_t blk = j.blocks[en.blk_off + i];
+    if (blk < 0) return false;
+    if (blk >= j.num_blocks) {
+        atomicCAS(j.err, 0, KVS_ERR_BOUNDS);
+        return false;
+    }
+    const uint64_t run_bytes = (uint64_t)ntok * j.row_bytes;
+    const uint64_t off = (uint64_t)k * j.piece_bytes;
+    if (off >= run_bytes) return false;
+    pc.len = (uint32_t)min((uint64_t)j.piece_bytes, run_bytes - off);
+    pc.chunk_addr = en.chunk + ((uint64_t)p * (uint64_t)en.n_tok + (uint64_t)first) * j.row_bytes + off;
+    pc.plane_addr = j.planes[p] + (uint64_t)blk * j.block_size * j.row_bytes + off;
+    return true;
+}
+
+// ---------------------------------------------------------------------------
+// Vector loads / stores.
+// ---------------------------------------------------------------------------
+template <int V> struct Vec;
+template <> struct Vec<16> { using T = uint4; };
+template <> struct Vec<8>  { using T = uint2; };
+template <> struct Vec<4>  { using T = uint32_t; };
+template <> struct Vec<2>  { using T = uint16_t; };
+template <> struct Vec<1>  { using T = uint8_t; };
+
+template <int V>
+__device__ __forceinline__ typename Vec<V>::T ld_stream(const typename Vec<V>::T* p) {
+    if constexpr (V == 16) {
+        uint4 r;
+        asm volatile("ld.global.nc.L1::no_allocate.v4.u32 {%0,%1,%2,%3}, [%4];"
+                     : "=r"(r.x), "=r"(r.y), "=r"(r.z), "=r"(r.w) : "l"(p));
+        return r;
+    } else {
+        return __ldg(p);
+    }
+}
+
+template <int V>
+__device__ __forceinline__ void st_stream(typename Vec<V>::T* p, const typename Vec<V>::T& v) {
+    if constexpr (V == 16) {
+        asm volatile("st.global.cs.v4.u32 [%0], {%1,%2,%3,%4};"
+                     :: "l"(p), "r"(v.x), "r"(v.y), "r"(v.z), "r"(v.w) : "memory");
+    } else {
+        *p = v;
+    }
+}
+
+template <int V>
+__device__ __forceinline__ bool vec_equal(const typename Vec<V>::T& a, const typename Vec<V>::T& b) {
+    if constexpr (V == 16) {
+        return a.x == b.x && a.y == b.y && a.z == b.z && a.w == b.w;
+    } else if constexpr (V == 8) {
+        return a.x == b.x && a.y == b.y;
+    } else {
+        return a == b;
+    }
+}
+
+// All threads of the CTA copy `len` bytes (a multiple of V) from src to dst:
+// U independent loads per thread are in flight before their stores.
+template <int V, int U>
+__device__ __forceinline__ void copy_piece(uint64_t src, uint64_t dst, uint32_t len) {
+    using T = typename Vec<V>::T;
+    const T* s = reinterpret_cast<const T*>(src);
+    T* d = reinterpret_cast<T*>(dst);
+    const uint32_t n = len / V;
+    const uint32_t stride = blockDim.x;
+    for (uint32_t base = threadIdx.x; base < n; base += stride * U) {
+        T r[U];
+#pragma unroll
+        for (int u = 0; u < U; ++u) {
+            const uint32_t k = base + u * stride;
+            if (k < n) r[u] = ld_stream<V>(s + k);
+        }
+#pragma unroll
+        for (int u = 0; u < U; ++u) {
+            const uint32_t k = base + u * stride;
+            if (k < n) st_stream<V>(d + k, r[u]);
+        }
+    }
+}
+
+template <int V, int U>
+__device__ __forceinline__ bool equal_piece(uint64_t a_addr, uint64_t b_addr, uint32_t len) {
+    using T = typename Vec<V>::T;
+    const T* a = reinterpret_cast<const T*>(a_addr);
+    const T* b = reinterpret_cast<const T*>(b_addr);
+    const uint32_t n = len / V;
+    bool same = true;
+    for (uint32_t k = threadIdx.x; k < n; k += blockDim.x)
+        same &= vec_equal<V>(ld_stream<V>(a + k), ld_stream<V>(b + k));
+    return same;
+}
+
+constexpr int kLdgThreads = 256;
+constexpr int kLdgUnroll = 8;
+
+template <int V, int MODE>
+__global__ void __launch_bounds__(kLdgThreads) kvs_ldg_kernel(const Decoder dc, uint32_t num_pieces) {
+    const Job& j = dc.job;
+    for (uint32_t q = blockIdx.x; q < num_pieces; q += gridDim.x) {
+        Piece pc;
+        if (!decode_piece(dc, q, pc)) continue;          // uniform across the CTA
+        if constexpr (MODE == MODE_RETRIEVE) {
+            copy_piece<V, kLdgUnroll>(pc.chunk_addr, pc.plane_addr, pc.len);
+        } else if constexpr (MODE == MODE_STORE) {
+            copy_piece<V, kLdgUnroll>(pc.plane_addr, pc.chunk_addr, pc.len);
+        } else {
+            if (!equal_piece<V, kLdgUnroll>(pc.chunk_addr, pc.plane_addr, pc.len))
+                atomicCAS(j.err, 0, KVS_ERR_ALIAS);
+        }
+    }
+}
+
+__global__ void __launch_bounds__(kLdgThreads) kvs_flat_copy_kernel(uint64_t dst, uint64_t src, uint64_t bytes) {
+    const uint64_t pieces = (bytes + kPieceBytes - 1) / kPieceBytes;
+    for (uint64_t q = blockIdx.x; q < pieces; q += gridDim.x) {
+        const uint64_t off = q * kPieceBytes;
+        const uint32_t len = (uint32_t)min((uint64_t)kPieceBytes, bytes - off);
+        copy_piece<16, kLdgUnroll>(src + off, dst + off, len);
+    }
+}
+
+// ---------------------------------------------------------------------------
+// TMA flavour: bulk async copies through a ring of shared-memory stages.
+// ---------------------------------------------------------------------------
+constexpr int kTmaStages = 6;
+constexpr uint64_t kWaitLimitNs = 2000000000ull;   // 2 s per wait: far above any piece
+
+__device__ __forceinline__ uint64_t global_ns() {
+    uint64_t t;
+    asm volatile("mov.u64 %0, %%globaltimer;" : "=l"(t));
+    return t;
+}
+
+__device__ __forceinline__ uint32_t smem_u32(const void* p) {
+    return (uint32_t)__cvta_generic_to_shared(p);
+}
+
+__device__ __forceinline__ void mbar_init(uint32_t bar, uint32_t count) {
+    asm volatile("mbarrier.init.shared::cta.b64 [%0], %1;" :: "r"(bar), "r"(count) : "memory");
+}
+
+__device__ __forceinline__ void mbar_expect_tx(uint32_t bar, uint32_t bytes) {
+    asm volatile("mbarrier.arrive.expect_tx.shared::cta.b64 _, [%0], %1;" :: "r"(bar), "r"(bytes) : "memory");
+}
+
+__device__ __forceinline__ bool mbar_try_wait(uint32_t bar, uint32_t parity) {
+    uint32_t ok;
+    asm volatile(
+        "{\n\t.reg .pred p;\n\t"
+        "mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2;\n\t"
+        "selp.u32 %0, 1, 0, p;\n\t}"
+        : "=r"(ok) : "r"(bar), "r"(parity) : "memory");
+    return ok != 0;
+}
+
+// Bounded wait: false once `limit_ns` has passed without the phase completing.
+__device__ __forceinline__ bool mbar_wait(uint32_t bar, uint32_t parity, uint64_t limit_ns) {
+    if (mbar_try_wait(bar, parity)) return true;
+    const uint64_t t0 = global_ns();
+    while (!mbar_try_wait(bar, parity)) {
+        if (global_ns() - t0 > limit_ns) return false;
+    }
+    return true;
+}
+
+__device__ __forceinline__ void bulk_load(uint32_t dst_smem, uint64_t src, uint32_t bytes, uint32_t bar) {
+    asm volatile(
+        "cp.async.bulk.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1], %2, [%3];"
+        :: "r"(dst_smem), "l"(src), "r"(bytes), "r"(bar) : "memory");
+}
+
+__device__ __forceinline__ void bulk_store(uint64_t dst, uint32_t src_smem, uint32_t bytes) {
+    asm volatile("cp.async.bulk.global.shared::cta.bulk_group [%0], [%1], %2;"
+                 :: "l"(dst), "r"(src_smem), "r"(bytes) : "memory");
+}
+
+__device__ __forceinline__ void bulk_commit() {
+    asm volatile("cp.async.bulk.commit_group;" ::: "memory");
+}
+
+template <int N>
+__device__ __forceinline__ void bulk_wait_read() {
+    asm volatile("cp.async.bulk.wait_group.read %0;" :: "n"(N) : "memory");
+}
+
+__device__ __forceinline__ void bulk_wait_all() {
+    asm volatile("cp.async.bulk.wait_group 0;" ::: "memory");
+}
+
+// One elected thread runs the whole pipeline: piece k of this CTA lives in
+// stage k % S; S-1 loads are kept in flight; before a stage is refilled the
+// bulk store that read it (one iteration earlier) must have finished reading.
+template <int S>
+__global__ void __launch_bounds__(32, 1) kvs_tma_kernel(const Decoder dc, uint32_t num_pieces) {
+    extern __shared__ __align__(128) uint8_t stage_mem[];
+    __shared__ __align__(8) uint64_t bars[S];
+    if (threadIdx.x != 0) return;
+    const Job& j = dc.job;
+    const uint32_t piece_bytes = j.piece_bytes;
+    const bool to_plane = (j.mode == MODE_RETRIEVE);
+
+    for (int s = 0; s < S; ++s) mbar_init(smem_u32(&bars[s]), 1);
+    asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+
+    uint32_t cursor = blockIdx.x;
+    auto next_piece = [&](Piece& out) -> bool {
+        while (cursor < num_pieces) {
+            const uint32_t q = cursor;
+            cursor += gridDim.x;
+            if (decode_piece(dc, q, out)) return true;
+        }
+        return false;
+    };
+    Piece pend[S] = {};
+    auto issue_load = [&](int s) {
+        const uint32_t bar = smem_u32(&bars[s]);
+        mbar_expect_tx(bar, pend[s].len);
+        bulk_load(smem_u32(stage_mem + (size_t)s * piece_bytes),
+                  to_plane ? pend[s].chunk_addr : pend[s].plane_addr, pend[s].len, bar);
+    };
+
+    uint32_t loaded = 0;
+    for (int s = 0; s < S - 1; ++s) {
+        if (!next_piece(pend[s])) break;
+        issue_load(s);
+        ++loaded;
+    }
+    for (uint32_t k = 0; k < loaded; ++k) {
+        const int s = (int)(k % S);
+        if (!mbar_wait(smem_u32(&bars[s]), (k / S) & 1u, kWaitLimitNs)) {
+            atomicCAS(j.err, 0, KVS_ERR_TIMEOUT);
+            // Let the loads still in flight land (bounded) before leaving.
+            for (uint32_t r = k; r < loaded; ++r)
+                mbar_wait(smem_u32(&bars[r % S]), (r / S) & 1u, kWaitLimitNs);
+            break;
+        }
+        bulk_store(to_plane ? pend[s].plane_addr : pend[s].chunk_addr,
+                   smem_u32(stage_mem + (size_t)s * piece_bytes), pend[s].len);
+        bulk_commit();
+        Piece nx;
+        if (next_piece(nx)) {
+            const int s2 = (int)((k + S - 1) % S);
+            bulk_wait_read<1>();
+            pend[s2] = nx;
+            issue_load(s2);
+            ++loaded;
+        }
+    }
+    bulk_wait_all();
+}
+
+// Waits on a barrier phase that nothing completes; the bounded wait must give up.
+__global__ void kvs_stall_kernel(int32_t* err, uint64_t limit_ns) {
+    __shared__ __align__(8) uint64_t bar;
+    if (threadIdx.x != 0) return;
+    mbar_init(smem_u32(&bar), 1);
+    asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+    if (!mbar_wait(smem_u32(&bar), 0, limit_ns)) atomicCAS(err, 0, KVS_ERR_TIMEOUT);
+}
+
+Decoder make_decoder(const Job& job) {
+    Decoder dc;
+    dc.job = job;
+    dc.ppr = make_fastdiv(job.pieces_per_run);
+    dc.bpc = make_fastdiv(job.blocks_per_chunk);
+    dc.planes = make_fastdiv(job.num_planes);
+    return dc;
+}
+
+int g_sms = 0;
+
+int num_sms() {
+    if (g_sms == 0) {
+        int dev = 0;
+        cudaGetDevice(&dev);
+        cudaDeviceGetAttribute(&g_sms, cudaDevAttrMultiProcessorCount, dev);
+        if (g_sms <= 0) g_sms = 1;
+    }
+    return g_sms;
+}
+
+int clamp_grid(int grid, int per_sm, uint64_t pieces) {
+    int full = num_sms() * per_sm;
+    if (grid <= 0 || grid > full) grid = full;
+    if ((uint64_t)grid > pieces) grid = (int)pieces;
+    return grid < 1 ? 1 : grid;
+}
+
+template <int V>
+cudaError_t launch_ldg_v(const Job& job, int grid, cudaStream_t s) {
+    grid = clamp_grid(grid, ldg_ctas_per_sm(), job.num_pieces);
+    const Decoder dc = make_decoder(job);
+    const uint32_t n = (uint32_t)job.num_pieces;
+    if (job.mode == MODE_RETRIEVE)
+        kvs_ldg_kernel<V, MODE_RETRIEVE><<<grid, kLdgThreads, 0, s>>>(dc, n);
+    else if (job.mode == MODE_STORE)
+        kvs_ldg_kernel<V, MODE_STORE><<<grid, kLdgThreads, 0, s>>>(dc, n);
+    else
+        kvs_ldg_kernel<V, MODE_COMPARE><<<grid, kLdgThreads, 0, s>>>(dc, n);
+    return cudaGetLastError();
+}
+
+}  // namespace
+
+int ldg_ctas_per_sm() {
+    static int n = 0;
+    if (n == 0) {
+        cudaOccupancyMaxActiveBlocksPerMultiprocessor(&n, kvs_ldg_kernel<16, MODE_RETRIEVE>, kLdgThreads, 0);
+        if (n <= 0) n = 1;
+        if (n > 4) n = 4;
+    }
+    return n;
+}
+
+int tma_ctas_per_sm() { return 1; }
+
+cudaError_t launch_ldg(const Job& job, int vec_bytes, int grid, cudaStream_t s) {
+    if (job.num_pieces == 0) return cudaSuccess;
+    switch (vec_bytes) {
+        case 16: return launch_ldg_v<16>(job, grid, s);
+        case 8:  return launch_ldg_v<8>(job, grid, s);
+        case 4:  return launch_ldg_v<4>(job, grid, s);
+        case 2:  return launch_ldg_v<2>(job, grid, s);
+        default: return launch_ldg_v<1>(job, grid, s);
+    }
+}
+
+cudaError_t launch_tma(const Job& job, int grid, cudaStream_t s) {
+    if (job.num_pieces == 0) return cudaSuccess;
+    const size_t smem = (size_t)kTmaStages * job.piece_bytes;
+    static size_t configured = 0;
+    if (configured < smem) {
+        cudaError_t e = cudaFuncSetAttribute(kvs_tma_kernel<kTmaStages>,
+                                             cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+        if (e != cudaSuccess) return e;
+        configured = smem;
+    }
+    grid = clamp_grid(grid, tma_ctas_per_sm(), job.num_pieces);
+    kvs_tma_kernel<kTmaStages><<<grid, 32, smem, s>>>(make_decoder(job), (uint32_t)job.num_pieces);
+    return cudaGetLastError();
+}
+
+cudaError_t launch_stall(int32_t* err, uint64_t limit_ns, cudaStream_t s) {
+    kvs_stall_kernel<<<1, 32, 0, s>>>(err, limit_ns);
+    return cudaGetLastError();
+}
+
+cudaError_t launch_flat_copy(void* dst, const void* src, uint64_t bytes, int grid, cudaStream_t s) {
+    const uint64_t pieces = (bytes + kPieceBytes - 1) / kPieceBytes;
+    if (pieces == 0) return cudaSuccess;
+    grid = clamp_grid(grid, ldg_ctas_per_sm(), pieces);
+    kvs_flat_copy_kernel<<<grid, kLdgThreads, 0, s>>>((uint64_t)dst, (uint64_t)src, bytes);
+    return cudaGetLastError();
+}
+
+}  // namespace kvs

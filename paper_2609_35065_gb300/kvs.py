@@ -1,0 +1,276 @@
+"""Python binding of the C ABI in ``include/kvs.h`` (ctypes; argument marshalling only).
+
+Every function has the C name and forwards to ``libkvs.so``; every byte is moved
+by the library's CUDA kernels or copy-engine transfers.  There is no fallback:
+if the library cannot be loaded, :func:`lib` raises.
+
+Buffers are passed as integer addresses or as objects with ``data_ptr()``
+(torch tensors).  Streams are passed as integer ``cudaStream_t`` handles,
+objects with ``cuda_stream`` (``torch.cuda.Stream``), or ``None`` / 0 for the
+legacy default stream.
+"""
+from __future__ import annotations
+
+import ctypes
+import os
+import threading
+from dataclasses import dataclass, field
+from typing import Sequence
+
+import numpy as np
+
+from . import build as _build
+
+# ---- constants mirrored from kvs.h ----------------------------------------
+KVS_OK = 0
+KVS_ERR_INVALID_ARG = -1
+KVS_ERR_BOUNDS = -2
+KVS_ERR_ALIAS = -3
+KVS_ERR_CUDA = -4
+KVS_ERR_TIMEOUT = -5
+KVS_ERR_NOMEM = -6
+KVS_ERR_UNSUPPORTED = -7
+ERROR_NAMES = {0: "KVS_OK", -1: "KVS_ERR_INVALID_ARG", -2: "KVS_ERR_BOUNDS", -3: "KVS_ERR_ALIAS",
+               -4: "KVS_ERR_CUDA", -5: "KVS_ERR_TIMEOUT", -6: "KVS_ERR_NOMEM", -7: "KVS_ERR_UNSUPPORTED"}
+
+KVS_SRC_HOST_PINNED = 1
+KVS_SRC_DEVICE = 2
+
+KVS_F_VALIDATE = 1 << 0
+KVS_F_FORCE_HOSTLINK = 1 << 1
+KVS_F_FORCE_HBMCOPY = 1 << 2
+KVS_F_FORCE_LDG = 1 << 3
+KVS_F_FORCE_TMA = 1 << 4
+KVS_F_NO_DEDUP = 1 << 5
+
+
+def KVS_F_MAX_CTAS(n: int) -> int:
+    return (int(n) & 0xFFFF) << 16
+
+
+KVS_VARIANT_HOSTLINK = 1
+KVS_VARIANT_HBMCOPY = 2
+KVS_KERNEL_LDG = 1
+KVS_KERNEL_TMA = 2
+
+EXPORTED = ("kvs_retrieve", "kvs_store", "kvs_query_bw", "kvs_get_choice", "kvs_check_errors",
+            "kvs_last_error", "kvs_shutdown", "kvs_version", "kvs_selftest_wait_timeout",
+            "kvs_stat_launches")
+
+
+class KvsError(RuntimeError):
+    def __init__(self, code: int, msg: str):
+        super().__init__(f"{ERROR_NAMES.get(code, code)}: {msg}")
+        self.code = code
+
+
+# ---- ctypes mirrors of the structs ----------------------------------------
+class kvs_geometry(ctypes.Structure):
+    _fields_ = [("num_layers", ctypes.c_int32), ("num_kv_heads", ctypes.c_int32),
+                ("head_dim", ctypes.c_int32), ("elem_bytes", ctypes.c_int32),
+                ("block_size", ctypes.c_int32), ("chunk_tokens", ctypes.c_int32)]
+
+
+class kvs_chunk(ctypes.Structure):
+    _fields_ = [("base", ctypes.c_void_p), ("num_tokens", ctypes.c_int32), ("residency", ctypes.c_int32)]
+
+
+class kvs_request(ctypes.Structure):
+    _fields_ = [("first_token", ctypes.c_int64), ("num_tokens", ctypes.c_int64),
+                ("chunks", ctypes.POINTER(kvs_chunk)), ("num_chunks", ctypes.c_int32),
+                ("block_table_len", ctypes.c_int32), ("block_table", ctypes.POINTER(ctypes.c_int32))]
+
+
+class kvs_paged_cache(ctypes.Structure):
+    _fields_ = [("kv_planes", ctypes.POINTER(ctypes.c_void_p)), ("num_blocks", ctypes.c_int64)]
+
+
+class kvs_bw_report(ctypes.Structure):
+    _fields_ = [("hbm_copy_gbs", ctypes.c_double), ("h2d_copy_engine_gbs", ctypes.c_double),
+                ("d2h_copy_engine_gbs", ctypes.c_double), ("zero_copy_read_gbs", ctypes.c_double),
+                ("zero_copy_write_gbs", ctypes.c_double), ("retrieve_gbs", ctypes.c_double * 2),
+                ("store_gbs", ctypes.c_double * 2), ("device_kernel_gbs", ctypes.c_double * 2),
+                ("chosen_retrieve_host", ctypes.c_int32), ("chosen_store_host", ctypes.c_int32),
+                ("chosen_kernel_device", ctypes.c_int32), ("num_sms", ctypes.c_int32),
+                ("probe_bytes", ctypes.c_int64)]
+
+    def as_dict(self) -> dict:
+        out = {}
+        for name, _ in self._fields_:
+            v = getattr(self, name)
+            out[name] = list(v) if isinstance(v, ctypes.Array) else v
+        return out
+
+
+# ---- library loading ------------------------------------------------------
+_lock = threading.Lock()
+_lib = None
+
+
+def lib_path() -> str:
+    return os.environ.get("KVS_LIBRARY", _build.LIB)
+
+
+def lib():
+    """Load ``libkvs.so`` (building it first if sources are newer).  Raises if impossible."""
+    global _lib
+    with _lock:
+        if _lib is None:
+            path = lib_path()
+            if "KVS_LIBRARY" not in os.environ and _build.stale():
+                _build.build_library()
+            if not os.path.exists(path):
+                raise ImportError(f"libkvs.so not found at {path}: build it with "
+                                  "`python -m paper_2609_35065_gb300.build`")
+            L = ctypes.CDLL(path)
+            P = ctypes.c_void_p
+            for name in ("kvs_retrieve", "kvs_store"):
+                fn = getattr(L, name)
+                fn.argtypes = [ctypes.POINTER(kvs_geometry), ctypes.POINTER(kvs_paged_cache),
+                               ctypes.POINTER(kvs_request), ctypes.c_int32, P, ctypes.c_uint32]
+                fn.restype = ctypes.c_int
+            L.kvs_query_bw.argtypes = [ctypes.POINTER(kvs_bw_report), P, ctypes.c_int64]
+            L.kvs_query_bw.restype = ctypes.c_int
+            L.kvs_get_choice.argtypes = [ctypes.POINTER(kvs_bw_report)]
+            L.kvs_get_choice.restype = ctypes.c_int
+            L.kvs_check_errors.argtypes = [P]
+            L.kvs_check_errors.restype = ctypes.c_int
+            L.kvs_last_error.argtypes = []
+            L.kvs_last_error.restype = ctypes.c_char_p
+            L.kvs_shutdown.argtypes = []
+            L.kvs_shutdown.restype = ctypes.c_int
+            L.kvs_version.argtypes = []
+            L.kvs_version.restype = ctypes.c_int
+            L.kvs_stat_launches.argtypes = []
+            L.kvs_stat_launches.restype = ctypes.c_int64
+            L.kvs_selftest_wait_timeout.argtypes = [P, ctypes.c_int64]
+            L.kvs_selftest_wait_timeout.restype = ctypes.c_int
+            _lib = L
+    return _lib
+
+
+# ---- marshalling helpers --------------------------------------------------
+def _addr(x) -> int:
+    if x is None:
+        return 0
+    if isinstance(x, int):
+        return x
+    if hasattr(x, "data_ptr"):
+        return int(x.data_ptr())
+    if isinstance(x, np.ndarray):
+        return int(x.ctypes.data)
+    raise TypeError(f"cannot take the address of {type(x)!r}")
+
+
+def _stream(s) -> int:
+    if s is None:
+        return 0
+    if isinstance(s, int):
+        return s
+    if hasattr(s, "cuda_stream"):
+        return int(s.cuda_stream)
+    raise TypeError(f"not a stream: {type(s)!r}")
+
+
+@dataclass
+class ChunkArg:
+    base: object                # address or tensor, [L][2][num_tokens][H][D]
+    num_tokens: int
+    residency: int = KVS_SRC_HOST_PINNED
+
+
+@dataclass
+class RequestArg:
+    block_table: np.ndarray     # int32 physical block ids (host)
+    chunks: Sequence[ChunkArg] = field(default_factory=list)
+    first_token: int = 0
+    num_tokens: int | None = None   # default: sum of chunk token counts
+
+
+def _geometry(g) -> kvs_geometry:
+    if isinstance(g, kvs_geometry):
+        return g
+    if hasattr(g, "layers"):
+        return kvs_geometry(g.layers, g.kv_heads, g.head_dim, g.elem_bytes, g.block_size, g.chunk_tokens)
+    return kvs_geometry(*g)
+
+
+class _Marshalled:
+    """Keeps every ctypes array alive for the duration of one C call."""
+
+    def __init__(self, planes, num_blocks, requests):
+        self.plane_arr = (ctypes.c_void_p * max(1, len(planes)))(*[_addr(p) for p in planes])
+        self.cache = kvs_paged_cache(ctypes.cast(self.plane_arr, ctypes.POINTER(ctypes.c_void_p)), int(num_blocks))
+        self.keep = []
+        self.reqs = (kvs_request * max(1, len(requests)))()
+        for k, r in enumerate(requests):
+            chunks = (kvs_chunk * max(1, len(r.chunks)))(
+                *[kvs_chunk(_addr(c.base), int(c.num_tokens), int(c.residency)) for c in r.chunks])
+            bt = np.ascontiguousarray(r.block_table, dtype=np.int32)
+            self.keep += [chunks, bt]
+            ntok = sum(int(c.num_tokens) for c in r.chunks) if r.num_tokens is None else int(r.num_tokens)
+            self.reqs[k] = kvs_request(int(r.first_token), ntok,
+                                       ctypes.cast(chunks, ctypes.POINTER(kvs_chunk)), len(r.chunks),
+                                       int(bt.size), bt.ctypes.data_as(ctypes.POINTER(ctypes.c_int32)))
+        self.n = len(requests)
+
+
+def _check(rc: int) -> int:
+    if rc != KVS_OK:
+        raise KvsError(rc, lib().kvs_last_error().decode(errors="replace"))
+    return rc
+
+
+# ---- the C ABI, same names ------------------------------------------------
+def kvs_retrieve(geom, planes, num_blocks, requests, stream=None, flags: int = 0) -> int:
+    """Enqueue retrieval of ``requests`` (list of :class:`RequestArg`) into the 2L
+    ``planes`` on ``stream``.  Raises :class:`KvsError` on a non-zero status."""
+    g = _geometry(geom)
+    m = _Marshalled(planes, num_blocks, requests)
+    return _check(lib().kvs_retrieve(ctypes.byref(g), ctypes.byref(m.cache), m.reqs, m.n,
+                                     _stream(stream), ctypes.c_uint32(flags)))
+
+
+def kvs_store(geom, planes, num_blocks, requests, stream=None, flags: int = 0) -> int:
+    """Enqueue store-back of ``requests`` from the planes into their chunk buffers."""
+    g = _geometry(geom)
+    m = _Marshalled(planes, num_blocks, requests)
+    return _check(lib().kvs_store(ctypes.byref(g), ctypes.byref(m.cache), m.reqs, m.n,
+                                  _stream(stream), ctypes.c_uint32(flags)))
+
+
+def kvs_query_bw(stream=None, probe_bytes: int = 0) -> dict:
+    rep = kvs_bw_report()
+    _check(lib().kvs_query_bw(ctypes.byref(rep), _stream(stream), int(probe_bytes)))
+    return rep.as_dict()
+
+
+def kvs_get_choice() -> dict:
+    rep = kvs_bw_report()
+    _check(lib().kvs_get_choice(ctypes.byref(rep)))
+    return rep.as_dict()
+
+
+def kvs_check_errors(stream=None) -> int:
+    return _check(lib().kvs_check_errors(_stream(stream)))
+
+
+def kvs_last_error() -> str:
+    return lib().kvs_last_error().decode(errors="replace")
+
+
+def kvs_shutdown() -> int:
+    return _check(lib().kvs_shutdown())
+
+
+def kvs_version() -> int:
+    return int(lib().kvs_version())
+
+
+def kvs_selftest_wait_timeout(stream=None, limit_ns: int = 50_000_000) -> int:
+    """Runs the bounded-wait self-test; returns the status code (KVS_ERR_TIMEOUT expected)."""
+    return int(lib().kvs_selftest_wait_timeout(_stream(stream), int(limit_ns)))
+
+
+def kvs_stat_launches() -> int:
+    return int(lib().kvs_stat_launches())

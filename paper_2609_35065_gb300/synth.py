@@ -45,6 +45,12 @@ class Request:
     residency: str = "host"             # fast-tier stand-in: "host" (pinned) or "device" (HBM)
     store_tokens: int = 0               # computed suffix stored back into chunks
     shared_prefix_tokens: int = 0       # leading tokens whose KV equals request 0's
+    first_token: int = 0                # start of the matched range (a multiple of chunk_tokens)
+    store_first: int | None = None      # start of the stored range (default: end of the match)
+
+    @property
+    def store_start(self) -> int:
+        return self.first_token + self.matched_tokens if self.store_first is None else self.store_first
 
 
 @dataclass
@@ -88,7 +94,7 @@ def tiny() -> Workload:
     with a seeded random permutation as block table."""
     g = Geometry(2, 4, 64)
     perm = _perm(128, 0)
-    reqs = [Request(512, 512, perm[:32].copy(), "host", store_tokens=512)]
+    reqs = [Request(512, 512, perm[:32].copy(), "host", store_tokens=512, store_first=0)]
     return Workload("tiny", g, 128, reqs, dist="uniform", seed=0)
 
 
@@ -159,12 +165,18 @@ def llama70b(requests: int = 4, prompt: int = 32768, buffer_frac: float = 1.0) -
 
 
 def custom(L, H, D, B, C, num_blocks, prompts, matched, seed=0, dist="uniform",
-           elem_bytes=2, residency="host") -> Workload:
-    """Small ad-hoc workload for tests: consecutive slices of one seeded permutation."""
+           elem_bytes=2, residency="host", firsts=None, store_tokens=None) -> Workload:
+    """Small ad-hoc workload for tests: consecutive slices of one seeded permutation.
+    ``residency`` is one value or one per request; ``firsts`` the matched-range starts."""
     g = Geometry(L, H, D, elem_bytes, B, C)
+    n = len(prompts)
+    res = [residency] * n if isinstance(residency, str) else list(residency)
+    firsts = [0] * n if firsts is None else list(firsts)
+    stores = [0] * n if store_tokens is None else list(store_tokens)
     nb = [-(-p // B) for p in prompts]
     tables = _consecutive_tables(_perm(num_blocks, seed), nb)
-    reqs = [Request(p, m, t, residency) for p, m, t in zip(prompts, matched, tables)]
+    reqs = [Request(p, m, t, rs, store_tokens=st, first_token=f)
+            for p, m, t, rs, f, st in zip(prompts, matched, tables, res, firsts, stores)]
     return Workload(f"custom_L{L}H{H}D{D}B{B}C{C}", g, num_blocks, reqs, dist=dist, seed=seed)
 
 
@@ -188,6 +200,24 @@ def fill_values(out, dist: str, generator) -> None:
         else:
             raise ValueError(dist)
         flat[at:at + n].copy_(v.to(torch.bfloat16).view(flat.dtype))
+
+
+def sentinel(elem_bytes: int) -> int:
+    """Sentinel element for any element size: the bf16 pattern repeated (0xA5 for bytes)."""
+    if elem_bytes == 1:
+        return 0xA5
+    return int.from_bytes(SENTINEL_BF16.to_bytes(2, "little") * (elem_bytes // 2), "little")
+
+
+def fill_bits(out, generator) -> None:
+    """Fill the torch tensor ``out`` with seeded random bits (non-bf16 element sizes)."""
+    import torch
+    flat = out.view(torch.uint8).view(-1)
+    step = 1 << 28
+    for at in range(0, flat.numel(), step):
+        n = min(step, flat.numel() - at)
+        flat[at:at + n].copy_(torch.randint(0, 256, (n,), generator=generator,
+                                            device=out.device, dtype=torch.int16).to(torch.uint8))
 
 
 def fill_values_np(out: np.ndarray, dist: str, seed: int) -> None:

@@ -1,0 +1,107 @@
+"""Element-by-element comparison of GPU results with the CPU oracle.
+
+Expected planes are built on the host from the same seeded inputs the GPU got
+(initial plane content + the oracle's retrieval of every request, one plane at
+a time so that tens-of-GB caches fit), then compared with the GPU plane copied
+back.  Nothing the GPU produced is ever fed to the oracle.
+"""
+from __future__ import annotations
+
+import os
+from concurrent.futures import ThreadPoolExecutor
+
+import numpy as np
+import torch
+
+import oracle
+from paper_2609_35065_gb300 import synth
+from paper_2609_35065_gb300.buffers import NP_DTYPES
+
+THREADS = min(8, os.cpu_count() or 1)
+
+
+def host_chunks(buf, which="chunks"):
+    """Host numpy views (copies for device chunks) of every request's chunk buffers."""
+    npd = NP_DTYPES[buf.workload.geom.elem_bytes]
+    out = []
+    for mine in getattr(buf, which):
+        out.append([(t.numpy() if t.device.type == "cpu" else t.cpu().numpy()).view(npd) for t in mine])
+    return out
+
+
+def expected_plane(buf, p, chunks_np):
+    w = buf.workload
+    g = w.geom
+    exp = buf.initial_plane(p)
+    planes = [None] * (2 * g.layers)
+    planes[p] = exp
+    for r, req in enumerate(w.requests):
+        if not chunks_np[r]:
+            continue
+        rc = oracle.retrieve(g.layers, g.kv_heads, g.head_dim, g.block_size, planes, w.num_blocks,
+                             req.first_token, chunks_np[r], req.block_table, p0=p, p1=p + 1)
+        assert rc == 0, rc
+    return exp
+
+
+def _diff(got, exp, label):
+    if np.array_equal(got, exp):
+        return None
+    idx = np.flatnonzero(got != exp)
+    return f"{label}: {idx.size} elements differ, first at {int(idx[0])} (got {got[idx[0]]:#x}, want {exp[idx[0]]:#x})"
+
+
+def check_retrieve(buf, planes=None, chunks_np=None):
+    """Every element of the listed planes (default: all) equals the oracle's result."""
+    g = buf.workload.geom
+    npd = NP_DTYPES[g.elem_bytes]
+    chunks_np = host_chunks(buf) if chunks_np is None else chunks_np
+    planes = range(2 * g.layers) if planes is None else planes
+
+    def one(p):
+        got = buf.planes[p].cpu().numpy().view(npd)
+        return _diff(got, expected_plane(buf, p, chunks_np), f"plane {p}")
+
+    with ThreadPoolExecutor(THREADS) as ex:
+        bad = [x for x in ex.map(one, planes) if x]
+    assert not bad, "\n".join(bad[:8])
+
+
+def check_store(buf, chunks_np=None):
+    """The GPU's store-back output equals the oracle's store from the oracle's planes."""
+    w = buf.workload
+    g = w.geom
+    npd = NP_DTYPES[g.elem_bytes]
+    chunks_np = host_chunks(buf) if chunks_np is None else chunks_np
+    fill = synth.sentinel(g.elem_bytes)
+    want = [[np.full(t.numel(), fill, dtype=npd) for t in mine] for mine in buf.store_chunks]
+
+    def one(p):
+        exp = expected_plane(buf, p, chunks_np)
+        planes = [None] * (2 * g.layers)
+        planes[p] = exp
+        for r, req in enumerate(buf.store_requests):
+            if not want[r]:
+                continue
+            rc = oracle.store(g.layers, g.kv_heads, g.head_dim, g.block_size, planes, w.num_blocks,
+                              req.first_token, want[r], req.block_table, p0=p, p1=p + 1)
+            assert rc == 0, rc
+
+    with ThreadPoolExecutor(THREADS) as ex:
+        list(ex.map(one, range(2 * g.layers)))
+    bad = []
+    for r, (mine, exp) in enumerate(zip(buf.store_chunks, want)):
+        for j, (t, e) in enumerate(zip(mine, exp)):
+            got = (t.numpy() if t.device.type == "cpu" else t.cpu().numpy()).view(npd)
+            d = _diff(got, e, f"store request {r} chunk {j}")
+            if d:
+                bad.append(d)
+    assert not bad, "\n".join(bad[:8])
+
+
+def free(buf):
+    for name in ("planes", "host_pool", "device_pool", "store_pool"):
+        setattr(buf, name, None)
+    buf.chunks = buf.store_chunks = []
+    buf.requests = buf.store_requests = []
+    torch.cuda.empty_cache()

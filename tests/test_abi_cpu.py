@@ -1,0 +1,97 @@
+"""The C-ABI library without a GPU: it builds, loads, exports every function
+declared in include/kvs.h, and rejects malformed calls before touching CUDA."""
+import ctypes
+import os
+import re
+
+import numpy as np
+import pytest
+
+from paper_2609_35065_gb300 import kvs
+
+ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+
+
+def declared_functions():
+    src = open(os.path.join(ROOT, "include", "kvs.h")).read()
+    src = re.sub(r"/\*.*?\*/", "", src, flags=re.S)
+    return sorted(set(re.findall(r"^\s*(?:const\s+)?\w+\s*\*?\s*(kvs_\w+)\s*\(", src, flags=re.M)))
+
+
+def test_library_exports_every_declared_function():
+    lib = kvs.lib()
+    names = declared_functions()
+    assert "kvs_retrieve" in names and "kvs_store" in names and "kvs_query_bw" in names
+    for n in names:
+        assert hasattr(lib, n), n
+    assert set(names) == set(kvs.EXPORTED)
+    assert kvs.kvs_version() == 10000
+
+
+def test_struct_layouts_match_header():
+    assert ctypes.sizeof(kvs.kvs_geometry) == 24
+    assert ctypes.sizeof(kvs.kvs_chunk) == 16
+    assert ctypes.sizeof(kvs.kvs_request) == 40
+    assert ctypes.sizeof(kvs.kvs_paged_cache) == 16
+    assert ctypes.sizeof(kvs.kvs_bw_report) == 5 * 8 + 6 * 8 + 4 * 4 + 8
+
+
+FAKE = 0x10000   # never dereferenced: every case below fails validation first
+G = (2, 2, 8, 2, 4, 8)
+
+
+def _req(tokens=(8, 8), table=(0, 1, 2, 3), first=0, res=kvs.KVS_SRC_HOST_PINNED, num_tokens=None):
+    chunks = [kvs.ChunkArg(FAKE + 4096 * i, n, res) for i, n in enumerate(tokens)]
+    return kvs.RequestArg(np.array(table, np.int32), chunks, first, num_tokens)
+
+
+def _code(fn=kvs.kvs_retrieve, geom=G, planes=None, nb=8, reqs=None, flags=0):
+    planes = [FAKE] * (2 * geom[0]) if planes is None else planes
+    reqs = [_req()] if reqs is None else reqs
+    with pytest.raises(kvs.KvsError) as ei:
+        fn(geom, planes, nb, reqs, None, flags)
+    return ei.value.code, str(ei.value)
+
+
+@pytest.mark.parametrize("fn", [kvs.kvs_retrieve, kvs.kvs_store])
+@pytest.mark.parametrize("case,code", [
+    (dict(geom=(0, 2, 8, 2, 4, 8)), kvs.KVS_ERR_INVALID_ARG),
+    (dict(geom=(2, 2, 8, 3, 4, 8)), kvs.KVS_ERR_INVALID_ARG),          # 3-byte elements
+    (dict(geom=(2, 2, 8, 2, 3, 8)), kvs.KVS_ERR_INVALID_ARG),          # C % B != 0
+    (dict(nb=0), kvs.KVS_ERR_INVALID_ARG),
+    (dict(planes=[FAKE, 0, FAKE, FAKE]), kvs.KVS_ERR_INVALID_ARG),
+    (dict(reqs=[_req(first=4)]), kvs.KVS_ERR_INVALID_ARG),             # not chunk-aligned
+    (dict(reqs=[_req(tokens=(4, 8))]), kvs.KVS_ERR_INVALID_ARG),       # partial chunk not last
+    (dict(reqs=[_req(tokens=(8, 9))]), kvs.KVS_ERR_INVALID_ARG),       # chunk larger than C
+    (dict(reqs=[_req(num_tokens=12)]), kvs.KVS_ERR_INVALID_ARG),       # chunks hold 16
+    (dict(reqs=[_req(res=7)]), kvs.KVS_ERR_INVALID_ARG),
+    (dict(reqs=[_req(table=(0, 1, 2))]), kvs.KVS_ERR_BOUNDS),          # table too short
+    (dict(reqs=[_req(table=(0, 1, 8, 3))]), kvs.KVS_ERR_BOUNDS),       # id >= num_blocks
+    (dict(reqs=[_req(table=(0, -1, 2, 3))]), kvs.KVS_ERR_BOUNDS),
+    (dict(flags=kvs.KVS_F_FORCE_HOSTLINK | kvs.KVS_F_FORCE_HBMCOPY), kvs.KVS_ERR_INVALID_ARG),
+    (dict(flags=kvs.KVS_F_FORCE_LDG | kvs.KVS_F_FORCE_TMA), kvs.KVS_ERR_INVALID_ARG),
+])
+def test_malformed_calls_are_rejected(fn, case, code):
+    got, msg = _code(fn=fn, **case)
+    assert got == code, msg
+    assert kvs.kvs_last_error() == msg.split(": ", 1)[1]
+
+
+def test_null_base_pointer_is_rejected():
+    r = _req()
+    r.chunks[0].base = 0
+    got, _ = _code(reqs=[r])
+    assert got == kvs.KVS_ERR_INVALID_ARG
+
+
+def test_call_too_large_is_rejected():
+    # 2^31 pieces or more: 32768 layers, B = 1, 128 chunks of 256 tokens
+    geom = (32768, 1, 8, 2, 1, 256)
+    reqs = [_req(tokens=(256,) * 128, table=tuple(range(256 * 128)))]
+    got, msg = _code(geom=geom, nb=256 * 128, reqs=reqs)
+    assert got == kvs.KVS_ERR_INVALID_ARG and "too large" in msg
+
+
+def test_empty_call_needs_no_device():
+    assert kvs.kvs_retrieve(G, [FAKE] * 4, 8, [], None, 0) == kvs.KVS_OK
+    assert kvs.kvs_store(G, [FAKE] * 4, 8, [_req(tokens=(), table=())], None, 0) == kvs.KVS_OK

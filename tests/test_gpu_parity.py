@@ -1,0 +1,228 @@
+"""GPU path (through the C ABI) against the CPU oracle, element by element.
+
+Small cases span several 32 KiB pieces, ragged last chunks, B = 1, rows that
+are not a multiple of 16 bytes, 1/2/4/8-byte elements, non-zero first tokens,
+both residencies and every variant flag.  Exact equality is required: the
+path only copies bytes.
+"""
+import numpy as np
+import pytest
+import torch
+
+import gpu_check as gc
+from paper_2609_35065_gb300 import buffers, kvs, synth
+
+pytestmark = pytest.mark.gpu
+
+VARIANTS = {
+    "default": 0,
+    "hostlink": kvs.KVS_F_FORCE_HOSTLINK,
+    "hbmcopy": kvs.KVS_F_FORCE_HBMCOPY,
+    "ldg": kvs.KVS_F_FORCE_LDG,
+    "tma": kvs.KVS_F_FORCE_TMA,
+    "hbmcopy_tma": kvs.KVS_F_FORCE_HBMCOPY | kvs.KVS_F_FORCE_TMA,
+    "few_ctas": kvs.KVS_F_MAX_CTAS(3),
+}
+
+
+@pytest.fixture(scope="module", autouse=True)
+def _cuda():
+    if not torch.cuda.is_available():
+        pytest.skip("no CUDA device")
+    torch.cuda.set_device(0)
+    yield
+    torch.cuda.synchronize()
+
+
+def _retrieve(buf, flags=0, stream=None):
+    w = buf.workload
+    kvs.kvs_retrieve(w.geom, buf.plane_ptrs, w.num_blocks, buf.requests, stream, flags | kvs.KVS_F_VALIDATE)
+
+
+def _store(buf, flags=0, stream=None):
+    w = buf.workload
+    kvs.kvs_store(w.geom, buf.plane_ptrs, w.num_blocks, buf.store_requests, stream, flags | kvs.KVS_F_VALIDATE)
+
+
+def test_wait_timeout_selftest_then_context_usable():
+    assert kvs.kvs_selftest_wait_timeout(None, 20_000_000) == kvs.KVS_ERR_TIMEOUT
+    assert kvs.kvs_check_errors(None) == kvs.KVS_OK
+    buf = buffers.allocate(synth.tiny(), store=True)
+    _retrieve(buf)
+    torch.cuda.synchronize()
+    gc.check_retrieve(buf)
+
+
+@pytest.mark.parametrize("variant", sorted(VARIANTS))
+def test_tiny_retrieve_then_store_round_trip(variant):
+    flags = VARIANTS[variant]
+    buf = buffers.allocate(synth.tiny(), store=True)
+    _retrieve(buf, flags)
+    torch.cuda.synchronize()
+    gc.check_retrieve(buf)
+    _store(buf, flags)
+    torch.cuda.synchronize()
+    gc.check_store(buf)
+    for a, b in zip(buf.chunks[0], buf.store_chunks[0]):        # store(retrieve(x)) == x
+        assert torch.equal(a, b)
+
+
+@pytest.mark.parametrize("variant", ["default", "hbmcopy", "tma"])
+def test_tiny_device_resident_source(variant):
+    w = synth.tiny()
+    w.requests[0].residency = "device"
+    buf = buffers.allocate(w, store=True, store_residency="device")
+    _retrieve(buf, VARIANTS[variant])
+    _store(buf, VARIANTS[variant])
+    torch.cuda.synchronize()
+    gc.check_retrieve(buf)
+    gc.check_store(buf)
+
+
+def _random_workload(seed):
+    rng = np.random.default_rng(seed)
+    e = int(rng.choice([1, 2, 2, 2, 4, 8]))
+    L = int(rng.integers(1, 5))
+    H = int(rng.integers(1, 9))
+    D = int(rng.choice([1, 3, 5, 8, 64, 128]))
+    B = int(rng.choice([1, 2, 8, 16, 32]))
+    C = B * int(rng.integers(1, 5))
+    nreq = int(rng.integers(1, 5))
+    prompts, matched, firsts, res, stores = [], [], [], [], []
+    for _ in range(nreq):
+        first = C * int(rng.integers(0, 2))
+        st = int(rng.integers(0, 2 * C + 1)) if rng.random() < 0.6 else 0
+        # a stored suffix starts where the match ends, so that end must be chunk-aligned
+        m = C * int(rng.integers(0, 5)) if st else int(rng.integers(0, 4 * C + 1))
+        prompts.append(first + m + st + int(rng.integers(0, B + 1)))
+        matched.append(m)
+        firsts.append(first)
+        res.append("device" if rng.random() < 0.4 else "host")
+        stores.append(st)
+    nb = sum(-(-p // B) for p in prompts) + int(rng.integers(0, 8))
+    w = synth.custom(L, H, D, B, C, nb, prompts, matched, seed=seed, elem_bytes=e,
+                     residency=res, firsts=firsts, store_tokens=stores)
+    return w
+
+
+@pytest.mark.parametrize("seed", range(24))
+def test_random_small_geometries(seed):
+    w = _random_workload(seed)
+    g = w.geom
+    flags_all = [0, kvs.KVS_F_FORCE_HOSTLINK, kvs.KVS_F_FORCE_HBMCOPY, kvs.KVS_F_FORCE_LDG,
+                 kvs.KVS_F_MAX_CTAS(1 + seed % 7)]
+    row = g.row_elems * g.elem_bytes
+    if row % 16 == 0:
+        flags_all.append(kvs.KVS_F_FORCE_TMA)
+    flags = flags_all[seed % len(flags_all)]
+    buf = buffers.allocate(w, store=True, store_residency="host" if seed % 2 else "device")
+    _retrieve(buf, flags)
+    _store(buf, flags)
+    torch.cuda.synchronize()
+    gc.check_retrieve(buf)
+    gc.check_store(buf)
+
+
+def test_tma_rejects_unaligned_rows():
+    w = synth.custom(1, 3, 5, 4, 8, 8, [16], [16])            # 30-byte rows
+    w.requests[0].residency = "device"
+    buf = buffers.allocate(w)
+    with pytest.raises(kvs.KvsError) as ei:
+        _retrieve(buf, kvs.KVS_F_FORCE_TMA)
+    assert ei.value.code == kvs.KVS_ERR_UNSUPPORTED
+    assert torch.all(buf.planes == buf.planes.view(-1)[0])     # nothing written
+
+
+def _shared(differ: bool):
+    # three requests whose first two blocks are shared physical blocks
+    g = synth.Geometry(2, 2, 8, 2, 4, 8)
+    perm = np.arange(40, dtype=np.int32)[::-1].copy()
+    t0 = perm[:6]
+    t1 = np.concatenate([t0[:2], perm[6:10]]).astype(np.int32)
+    t2 = np.concatenate([t0[:2], perm[10:12]]).astype(np.int32)
+    reqs = [synth.Request(24, 24, t0, "host", shared_prefix_tokens=0),
+            synth.Request(24, 24, t1, "device", shared_prefix_tokens=8),
+            synth.Request(16, 12, t2, "host", shared_prefix_tokens=8)]
+    w = synth.Workload("shared", g, 40, reqs, dist="uniform", seed=3)
+    buf = buffers.allocate(w)
+    if differ:
+        buf.chunks[2][0].view(4, 8, 16)[:, 1, :] += 1          # token 1 of request 2 differs
+    return buf
+
+
+@pytest.mark.parametrize("flags", [0, kvs.KVS_F_NO_DEDUP, kvs.KVS_F_FORCE_HBMCOPY])
+def test_shared_blocks_written_once_with_equal_content(flags):
+    buf = _shared(differ=False)
+    _retrieve(buf, flags)
+    torch.cuda.synchronize()
+    gc.check_retrieve(buf)
+
+
+def test_shared_blocks_with_differing_bytes_are_reported():
+    buf = _shared(differ=True)
+    with pytest.raises(kvs.KvsError) as ei:
+        _retrieve(buf)
+    assert ei.value.code == kvs.KVS_ERR_ALIAS
+    assert kvs.kvs_check_errors(None) == kvs.KVS_OK            # the word was cleared
+
+
+def test_block_named_twice_in_one_request_is_alias():
+    w = synth.custom(1, 1, 8, 2, 4, 8, [8], [8])
+    w.requests[0].block_table[1] = w.requests[0].block_table[0]
+    buf = buffers.allocate(w)
+    with pytest.raises(kvs.KvsError) as ei:
+        _retrieve(buf)
+    assert ei.value.code == kvs.KVS_ERR_ALIAS
+
+
+def test_out_of_range_block_is_rejected_before_any_write():
+    w = synth.custom(2, 2, 8, 4, 8, 8, [16], [16])
+    w.requests[0].block_table[3] = 8
+    buf = buffers.allocate(w)
+    with pytest.raises(kvs.KvsError) as ei:
+        _retrieve(buf)
+    assert ei.value.code == kvs.KVS_ERR_BOUNDS
+    torch.cuda.synchronize()
+    assert torch.all(buf.planes == buf.planes.view(-1)[0])
+
+
+def test_empty_calls_touch_nothing():
+    w = synth.custom(2, 2, 8, 4, 8, 8, [16, 8], [0, 0])
+    buf = buffers.allocate(w)
+    _retrieve(buf)
+    kvs.kvs_retrieve(w.geom, buf.plane_ptrs, w.num_blocks, [], None, kvs.KVS_F_VALIDATE)
+    torch.cuda.synchronize()
+    assert torch.all(buf.planes == buf.planes.view(-1)[0])
+
+
+def test_streams_and_async_host_arrays():
+    """The call returns before the copy runs; its host arrays may be dropped at once."""
+    buf = buffers.allocate(synth.tiny())
+    s = torch.cuda.Stream()
+    w = buf.workload
+    reqs = [kvs.RequestArg(r.block_table.copy(), list(r.chunks)) for r in buf.requests]
+    kvs.kvs_retrieve(w.geom, buf.plane_ptrs, w.num_blocks, reqs, s, 0)
+    for r in reqs:
+        r.block_table[:] = -7                                   # reuse the host arrays
+    s.synchronize()
+    assert kvs.kvs_check_errors(s) == kvs.KVS_OK
+    gc.check_retrieve(buf)
+
+
+def test_query_bw_reports_and_chooses():
+    rep = kvs.kvs_query_bw(None, 256 << 20)
+    for k in ("hbm_copy_gbs", "h2d_copy_engine_gbs", "d2h_copy_engine_gbs",
+              "zero_copy_read_gbs", "zero_copy_write_gbs"):
+        assert rep[k] > 1.0, (k, rep)
+    assert rep["chosen_retrieve_host"] in (kvs.KVS_VARIANT_HOSTLINK, kvs.KVS_VARIANT_HBMCOPY)
+    assert rep["chosen_kernel_device"] in (kvs.KVS_KERNEL_LDG, kvs.KVS_KERNEL_TMA)
+    assert rep["num_sms"] > 0
+    got = kvs.kvs_get_choice()
+    assert got["chosen_retrieve_host"] == rep["chosen_retrieve_host"]
+    # the chosen defaults still give exact results
+    buf = buffers.allocate(synth.tiny(), store=True)
+    _retrieve(buf)
+    _store(buf)
+    torch.cuda.synchronize()
+    gc.check_retrieve(buf)
+    gc.check_store(buf)

@@ -1,0 +1,103 @@
+"""Full-size workloads through the C ABI, compared with the CPU oracle on every
+element of every plane (streamed one plane at a time through the oracle)."""
+import numpy as np
+import pytest
+import torch
+
+import gpu_check as gc
+from paper_2609_35065_gb300 import buffers, kvs, synth
+
+pytestmark = pytest.mark.gpu
+
+
+@pytest.fixture(scope="module", autouse=True)
+def _cuda():
+    if not torch.cuda.is_available():
+        pytest.skip("no CUDA device")
+    torch.cuda.set_device(0)
+    yield
+    torch.cuda.empty_cache()
+
+
+def _run(buf, fn="retrieve", flags=0):
+    w = buf.workload
+    reqs = buf.requests if fn == "retrieve" else buf.store_requests
+    getattr(kvs, f"kvs_{fn}")(w.geom, buf.plane_ptrs, w.num_blocks, reqs, None, flags | kvs.KVS_F_VALIDATE)
+
+
+@pytest.mark.parametrize("flags", [0, kvs.KVS_F_FORCE_HOSTLINK, kvs.KVS_F_FORCE_HBMCOPY],
+                         ids=["default", "hostlink", "hbmcopy"])
+def test_llama8b_host_source(flags):
+    buf = buffers.allocate(synth.llama8b())
+    assert buf.payload_bytes == 4 << 30
+    _run(buf, flags=flags)
+    torch.cuda.synchronize()
+    gc.check_retrieve(buf)
+    gc.free(buf)
+
+
+@pytest.mark.parametrize("ratio", [25, 50, 75])
+def test_sweep_mixed_residency(ratio):
+    w = synth.sweep(ratio / 100)
+    res = {r.residency for r in w.requests}
+    assert res == {"host", "device"}
+    buf = buffers.allocate(w)
+    _run(buf)
+    torch.cuda.synchronize()
+    gc.check_retrieve(buf)
+    gc.free(buf)
+
+
+def test_qwen14b_shared_prefix_retrieve_and_suffix_store():
+    w = synth.qwen14b()
+    assert w.notes["shared_blocks"] == 76
+    buf = buffers.allocate(w, store=True, store_residency="host", plane_init="random")
+    _run(buf, "retrieve")
+    _run(buf, "store")
+    torch.cuda.synchronize()
+    chunks_np = gc.host_chunks(buf)
+    gc.check_retrieve(buf, chunks_np=chunks_np)
+    gc.check_store(buf, chunks_np=chunks_np)
+    gc.free(buf)
+
+
+def test_qwen14b_store_to_hbm_destination_hbmcopy_path():
+    w = synth.qwen14b()
+    buf = buffers.allocate(w, store=True, store_residency="device", plane_init="random")
+    _run(buf, "retrieve", kvs.KVS_F_FORCE_HBMCOPY)
+    _run(buf, "store", kvs.KVS_F_FORCE_TMA)
+    torch.cuda.synchronize()
+    chunks_np = gc.host_chunks(buf)
+    gc.check_retrieve(buf, chunks_np=chunks_np)
+    gc.check_store(buf, chunks_np=chunks_np)
+    gc.free(buf)
+
+
+def test_llama70b_quarter_buffer_refilled_between_passes():
+    """Pinned fast-tier buffer holds 25% of the batch: 4 passes, refilled in between."""
+    w = synth.llama70b(buffer_frac=0.25)
+    g = w.geom
+    per_tok = 2 * g.layers * g.row_elems
+    n = w.num_blocks * g.block_size * g.row_elems
+    planes = torch.full((2 * g.layers, n), synth.SENTINEL_BF16, dtype=torch.int16, device="cuda")
+    one_req = w.requests[0].matched_tokens * per_tok
+    pinned = torch.empty(one_req, dtype=torch.int16, pin_memory=True)
+    assert pinned.numel() * 2 * len(w.requests) == w.matched_tokens * per_tok * 2
+    host_copies = []
+    for k, r in enumerate(w.requests):
+        gen = torch.Generator(device="cuda").manual_seed(100 + k)
+        tmp = torch.empty(one_req, dtype=torch.int16, device="cuda")
+        synth.fill_values(tmp, "normal", gen)
+        torch.cuda.synchronize()
+        pinned.copy_(tmp)                                   # refill between passes (untimed)
+        del tmp
+        chunks = [pinned[j * 256 * per_tok:(j + 1) * 256 * per_tok] for j in range(r.matched_tokens // 256)]
+        req = kvs.RequestArg(r.block_table, [kvs.ChunkArg(c, 256) for c in chunks])
+        kvs.kvs_retrieve(g, [int(planes[p].data_ptr()) for p in range(2 * g.layers)], w.num_blocks,
+                         [req], None, kvs.KVS_F_VALIDATE)
+        torch.cuda.synchronize()
+        host_copies.append([c.numpy().copy().view(np.uint16) for c in chunks])
+    fake = buffers.Buffers(w, planes, [], [], [], [])
+    gc.check_retrieve(fake, chunks_np=host_copies)
+    del planes, pinned
+    torch.cuda.empty_cache()
