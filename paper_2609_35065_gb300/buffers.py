@@ -169,6 +169,6 @@ def allocate(w: synth.Workload, device: str = "cuda", store: bool = False,
                 off += n * per_tok
             store_chunks.append(mine)
             store_requests.append(RequestArg(r.block_table, [ChunkArg(t, t.numel() // per_tok, res) for t in mine],
-                                             first_token=r.store_start))
+                                             first_token=r.store_start if r.store_tokens else 0))
     return Buffers(w, planes, chunks, store_chunks, requests, store_requests,
                    host_pool, device_pool, store_pool, plane_init)
