@@ -209,6 +209,40 @@ int kvs_selftest_wait_timeout(void* cuda_stream, int64_t limit_ns);
 /* Number of kernels this library has launched in this process (all devices). */
 int64_t kvs_stat_launches(void);
 
+/*
+ * Retrieval that allocates nothing.  The paper has no counterpart: this entry
+ * point exists for callers that cannot let a library allocate GPU memory --
+ * serving runtimes that reserve almost all free HBM for their own KV block
+ * pool at start-up and sub-allocate it themselves (a cudaMalloc during serving
+ * could fail or break their accounting), and latency-critical paths where
+ * cudaMalloc / cudaFree would synchronise the device.
+ *
+ * Same arguments and result as kvs_retrieve, with these differences:
+ *  - no cudaMalloc, cudaFree, cudaHostAlloc or other allocating call is made;
+ *    the kernel's scratch (descriptor tables and error word) lives in a static
+ *    device array of KVS_NOALLOC_SCRATCH_BYTES compiled into the library,
+ *    which every GPU that loads the library holds until the process exits.
+ *    A call whose tables do not fit (about 10 KB for 16 requests of 2048
+ *    tokens at 32 layers; roughly 16 + 4 * chunk_tokens / block_size bytes
+ *    per chunk, twice the block part with KVS_F_VALIDATE) returns
+ *    KVS_ERR_UNSUPPORTED with a message saying so;
+ *  - the first call on a device looks up the device address of that array
+ *    (once per device, with that device current); make that first call
+ *    before any stream capture;
+ *  - every call shares the one array and overwrites it: calls whose work can
+ *    overlap on the GPU (different streams, or other host threads) race and
+ *    must be ordered by the caller; the error word is cleared at the start of
+ *    each call;
+ *  - host chunks are always read directly over the host link and every chunk
+ *    is moved by the vector-load kernel (KVS_F_FORCE_HBMCOPY, KVS_F_FORCE_TMA
+ *    and KVS_F_NO_DEDUP are refused with KVS_ERR_UNSUPPORTED);
+ *  - device-side errors are only reported with KVS_F_VALIDATE.
+ */
+#define KVS_NOALLOC_SCRATCH_BYTES (1u << 20)
+int kvs_retrieve_noalloc(const kvs_geometry* geom, const kvs_paged_cache* cache,
+                         const kvs_request* requests, int32_t num_requests,
+                         void* cuda_stream, uint32_t flags);
+
 /* ABI version of this header: major * 10000 + minor * 100 + patch. */
 int kvs_version(void);
 #define KVS_VERSION 10000

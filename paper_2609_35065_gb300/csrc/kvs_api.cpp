@@ -679,6 +679,9 @@ int query_bw(DevState& st, kvs_bw_report* out, cudaStream_t s, int64_t probe_byt
 }
 
 }  // namespace
+
+void set_last_error(const char* msg) { t_error = msg; }
+
 }  // namespace kvs
 
 using namespace kvs;

@@ -53,6 +53,8 @@ cudaError_t launch_flat_copy(void* dst, const void* src, uint64_t bytes, int gri
 // One CTA waits (bounded by limit_ns) on an mbarrier phase that nothing
 // completes, then records KVS_ERR_TIMEOUT: exercises the bounded-wait path.
 cudaError_t launch_stall(int32_t* err, uint64_t limit_ns, cudaStream_t s);
+// Sets the calling thread's message returned by kvs_last_error() (kvs_api.cpp).
+void set_last_error(const char* msg);
 // CTAs per SM the flavour runs with (occupancy); used to size persistent grids.
 int ldg_ctas_per_sm();
 int tma_ctas_per_sm();

@@ -55,7 +55,8 @@ KVS_KERNEL_TMA = 2
 
 EXPORTED = ("kvs_retrieve", "kvs_store", "kvs_query_bw", "kvs_get_choice", "kvs_check_errors",
             "kvs_last_error", "kvs_shutdown", "kvs_version", "kvs_selftest_wait_timeout",
-            "kvs_stat_launches")
+            "kvs_stat_launches", "kvs_retrieve_noalloc")
+KVS_NOALLOC_SCRATCH_BYTES = 1 << 20
 
 
 class KvsError(RuntimeError):
@@ -124,7 +125,7 @@ def lib():
                                   "`python -m paper_2609_35065_gb300.build`")
             L = ctypes.CDLL(path)
             P = ctypes.c_void_p
-            for name in ("kvs_retrieve", "kvs_store"):
+            for name in ("kvs_retrieve", "kvs_store", "kvs_retrieve_noalloc"):
                 fn = getattr(L, name)
                 fn.argtypes = [ctypes.POINTER(kvs_geometry), ctypes.POINTER(kvs_paged_cache),
                                ctypes.POINTER(kvs_request), ctypes.c_int32, P, ctypes.c_uint32]
@@ -274,3 +275,13 @@ def kvs_selftest_wait_timeout(stream=None, limit_ns: int = 50_000_000) -> int:
 
 def kvs_stat_launches() -> int:
     return int(lib().kvs_stat_launches())
+
+
+def kvs_retrieve_noalloc(geom, planes, num_blocks, requests, stream=None, flags: int = 0) -> int:
+    """Like :func:`kvs_retrieve`, for callers that cannot let the library allocate GPU
+    memory: its scratch is a static device array of KVS_NOALLOC_SCRATCH_BYTES, so the
+    call allocates nothing; calls that overlap on the GPU race on that array."""
+    g = _geometry(geom)
+    m = _Marshalled(planes, num_blocks, requests)
+    return _check(lib().kvs_retrieve_noalloc(ctypes.byref(g), ctypes.byref(m.cache), m.reqs, m.n,
+                                             _stream(stream), ctypes.c_uint32(flags)))
