@@ -135,6 +135,9 @@ typedef struct kvs_paged_cache {
  * token i of the chunk, head h and dim d,
  *     plane[2l+kv][slot(s_j + i)][h][d] = chunk_j[l][kv][i][h][d],
  * with s_j the first request token of chunk j.  Nothing else is written.
+ * When a call holds both device- and host-resident chunks, the two classes
+ * are copied concurrently (the device part on a library stream that joins
+ * the caller's stream before the call's work is complete).
  * A physical block named by several requests (a shared prefix) must carry the
  * same KV in each; it is written once, from the request that covers the most
  * of its tokens (the lowest index among equals), unless KVS_F_NO_DEDUP.
@@ -168,14 +171,18 @@ typedef struct kvs_bw_report {
     int32_t chosen_store_host;     /* KVS_VARIANT_* used for host chunks by kvs_store      */
     int32_t chosen_kernel_device;  /* KVS_KERNEL_* used for device-resident chunks         */
     int32_t num_sms;
+    int32_t hostlink_ctas;         /* CTAs given to host-link retrieval kernels (0 = all): the
+                                      smallest probed grid within 0.5% of the best rate, so
+                                      that kernels on other streams keep the remaining SMs */
+    int32_t store_ctas;            /* the same for host-link store kernels                 */
     int64_t probe_bytes;           /* bytes moved per probe                                */
 } kvs_bw_report;
 
 /*
  * Measures the bandwidths above on the current device with probes of
  * probe_bytes bytes (0 = 1 GiB), synchronously, using cuda_stream, and makes
- * the measured fastest variants the defaults of later kvs_retrieve / kvs_store
- * calls on this device.  Allocates (and frees before returning) probe
+ * the measured fastest variants (and the host-link CTA caps) the defaults of
+ * later kvs_retrieve / kvs_store calls on this device.  Allocates (and frees before returning) probe
  * buffers: 2 * probe_bytes of device memory and probe_bytes of pinned host
  * memory.  `out` may be NULL.
  */
@@ -245,7 +252,7 @@ int kvs_retrieve_noalloc(const kvs_geometry* geom, const kvs_paged_cache* cache,
 
 /* ABI version of this header: major * 10000 + minor * 100 + patch. */
 int kvs_version(void);
-#define KVS_VERSION 10000
+#define KVS_VERSION 10100
 
 #ifdef __cplusplus
 }

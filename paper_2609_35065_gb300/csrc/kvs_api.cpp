@@ -73,6 +73,9 @@ struct DevState {
     cudaEvent_t  ring_filled[kRingSlots] = {};
     cudaEvent_t  ring_free[kRingSlots] = {};
     cudaEvent_t  ev_fork = nullptr, ev_join = nullptr;
+    // device-resident chunks run on this stream, beside the host-resident ones
+    cudaStream_t aux_stream = nullptr;
+    cudaEvent_t  ev_aux_fork = nullptr, ev_aux_join = nullptr;
     // per-block ownership for de-duplication: stamp[b] == gen -> owner[b] valid
     std::vector<uint32_t> stamp;
     std::vector<int64_t>  owner;
@@ -81,6 +84,8 @@ struct DevState {
     int          retrieve_host = KVS_VARIANT_HOSTLINK;
     int          store_host = KVS_VARIANT_HOSTLINK;
     int          kernel_device = KVS_KERNEL_LDG;
+    int          hostlink_ctas = 0;          // CTA cap of host-link kernels, 0 = whole GPU
+    int          store_ctas = 0;
     kvs_bw_report report{};
 };
 
@@ -107,6 +112,9 @@ int get_state(DevState** out) {
         }
         KVS_CUDA(cudaEventCreateWithFlags(&st.ev_fork, cudaEventDisableTiming));
         KVS_CUDA(cudaEventCreateWithFlags(&st.ev_join, cudaEventDisableTiming));
+        KVS_CUDA(cudaStreamCreateWithFlags(&st.aux_stream, cudaStreamNonBlocking));
+        KVS_CUDA(cudaEventCreateWithFlags(&st.ev_aux_fork, cudaEventDisableTiming));
+        KVS_CUDA(cudaEventCreateWithFlags(&st.ev_aux_join, cudaEventDisableTiming));
         st.report.num_sms = st.sms;
         st.report.chosen_retrieve_host = st.retrieve_host;
         st.report.chosen_store_host = st.store_host;
@@ -529,12 +537,24 @@ int copy_call(const kvs_geometry* g, const kvs_paged_cache* cache, const kvs_req
                                                                     : (retrieve ? st.retrieve_host : st.store_host);
     const Mode mode = retrieve ? MODE_RETRIEVE : MODE_STORE;
 
+    const int host_grid = grid ? grid : (retrieve ? st.hostlink_ctas : st.store_ctas);
+
     Uploaded u;
     rc = upload(st, pl, s, u);
     if (rc) return rc;
+    // With both classes present, the HBM-bound device part runs on the aux
+    // stream while the link-bound host part runs on the caller's stream.
+    const bool fork = pl.num_device && pl.num_host;
     if (pl.num_device) {
-        rc = launch_kernel(make_job(st, g, cache, pl, u, 0, pl.num_device, mode), flavour, vec, grid, s);
+        cudaStream_t ds = s;
+        if (fork) {
+            KVS_CUDA(cudaEventRecord(st.ev_aux_fork, s));
+            KVS_CUDA(cudaStreamWaitEvent(st.aux_stream, st.ev_aux_fork, 0));
+            ds = st.aux_stream;
+        }
+        rc = launch_kernel(make_job(st, g, cache, pl, u, 0, pl.num_device, mode), flavour, vec, grid, ds);
         if (rc) return rc;
+        if (fork) KVS_CUDA(cudaEventRecord(st.ev_aux_join, st.aux_stream));
     }
     if (pl.num_host) {
         if (host_variant == KVS_VARIANT_HBMCOPY) {
@@ -544,10 +564,11 @@ int copy_call(const kvs_geometry* g, const kvs_paged_cache* cache, const kvs_req
             rc = run_hbmcopy(st, g, cache, pl, u, mode, flavour, grid, s, host_addr);
         } else {
             rc = launch_kernel(make_job(st, g, cache, pl, u, pl.num_device, pl.num_host, mode),
-                               KVS_KERNEL_LDG, vec, grid, s);
+                               KVS_KERNEL_LDG, vec, host_grid, s);
         }
         if (rc) return rc;
     }
+    if (fork) KVS_CUDA(cudaStreamWaitEvent(s, st.ev_aux_join, 0));
     if (!pl.blocks_cmp.empty()) {
         Job j = make_job(st, g, cache, pl, u, 0, (uint32_t)pl.entries.size(), MODE_COMPARE);
         j.blocks = u.blocks_cmp;
@@ -591,6 +612,7 @@ int query_bw(DevState& st, kvs_bw_report* out, cudaStream_t s, int64_t probe_byt
     kvs_bw_report rep{};
     rep.num_sms = st.sms;
     rep.probe_bytes = probe_bytes;
+    st.hostlink_ctas = st.store_ctas = 0;          // variant probes below use the whole GPU
     uint8_t *d0 = nullptr, *d1 = nullptr, *h = nullptr;
     auto cleanup = [&]() {
         if (d0) cudaFree(d0);
@@ -664,9 +686,31 @@ int query_bw(DevState& st, kvs_bw_report* out, cudaStream_t s, int64_t probe_byt
         cleanup();
         return rc;
     }
+    // Smallest host-link grid within 0.5% of the best: a grid that fills every SM
+    // buys nothing once the link is saturated and starves concurrent kernels.
+    {
+        const int full = st.sms * ldg_ctas_per_sm();
+        const int cand[] = {16, 24, 32, 48, 64, 96, 128, full};
+        double gb[2][8] = {};
+        for (int dir = 0; dir < 2; ++dir) {
+            double best = 0;
+            for (int k = 0; k < 8; ++k) {
+                rc = probe_call(&rh, dir == 0, KVS_F_FORCE_HOSTLINK | KVS_F_MAX_CTAS(cand[k]), &gb[dir][k]);
+                if (rc) { cleanup(); return rc; }
+                best = std::max(best, gb[dir][k]);
+            }
+            int pick = 0;
+            for (int k = 0; k < 8; ++k)
+                if (gb[dir][k] >= 0.995 * best) { pick = cand[k]; break; }
+            if (pick >= full) pick = 0;
+            if (dir == 0) rep.hostlink_ctas = pick; else rep.store_ctas = pick;
+        }
+    }
 #undef PROBE
     KVS_CUDA(cudaStreamSynchronize(s));
     cleanup();
+    st.hostlink_ctas = rep.hostlink_ctas;
+    st.store_ctas = rep.store_ctas;
     st.retrieve_host = rep.retrieve_gbs[1] > rep.retrieve_gbs[0] ? KVS_VARIANT_HBMCOPY : KVS_VARIANT_HOSTLINK;
     st.store_host = rep.store_gbs[1] > rep.store_gbs[0] ? KVS_VARIANT_HBMCOPY : KVS_VARIANT_HOSTLINK;
     st.kernel_device = rep.device_kernel_gbs[1] > rep.device_kernel_gbs[0] ? KVS_KERNEL_TMA : KVS_KERNEL_LDG;
@@ -723,6 +767,8 @@ int kvs_get_choice(kvs_bw_report* out) {
     out->chosen_store_host = st->store_host;
     out->chosen_kernel_device = st->kernel_device;
     out->num_sms = st->sms;
+    out->hostlink_ctas = st->hostlink_ctas;
+    out->store_ctas = st->store_ctas;
     return KVS_OK;
 }
 
@@ -756,6 +802,9 @@ int kvs_shutdown(void) {
         }
         cudaEventDestroy(st.ev_fork);
         cudaEventDestroy(st.ev_join);
+        cudaEventDestroy(st.ev_aux_fork);
+        cudaEventDestroy(st.ev_aux_join);
+        if (st.aux_stream) cudaStreamDestroy(st.aux_stream);
         if (st.ring) cudaFree(st.ring);
         if (st.copy_stream) cudaStreamDestroy(st.copy_stream);
         if (st.err) cudaFree(st.err);

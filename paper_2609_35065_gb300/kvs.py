@@ -93,6 +93,7 @@ class kvs_bw_report(ctypes.Structure):
                 ("store_gbs", ctypes.c_double * 2), ("device_kernel_gbs", ctypes.c_double * 2),
                 ("chosen_retrieve_host", ctypes.c_int32), ("chosen_store_host", ctypes.c_int32),
                 ("chosen_kernel_device", ctypes.c_int32), ("num_sms", ctypes.c_int32),
+                ("hostlink_ctas", ctypes.c_int32), ("store_ctas", ctypes.c_int32),
                 ("probe_bytes", ctypes.c_int64)]
 
     def as_dict(self) -> dict:

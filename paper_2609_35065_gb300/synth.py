@@ -98,16 +98,17 @@ def tiny() -> Workload:
     return Workload("tiny", g, 128, reqs, dist="uniform", seed=0)
 
 
-def llama8b(requests: int = 16, prompt: int = 4096, hit: float = 0.5) -> Workload:
+def llama8b(requests: int = 16, prompt: int = 4096, hit: float = 0.5, num_blocks: int = 20000) -> Workload:
     """Llama-3-8B-shaped KV (32 layers, 8 KV heads, head_dim 128, 128 KiB/token),
     16 requests of 4096-token prompts at 50% prefix hit, 20,000-block cache with
     seeded random free-block assignment; source in pinned host memory."""
     g = Geometry(32, 8, 128)
     nb_each = -(-prompt // g.block_size)
-    tables = _consecutive_tables(_perm(20000, 0), [nb_each] * requests)
+    tables = _consecutive_tables(_perm(num_blocks, 0), [nb_each] * requests)
     matched = int(prompt * hit) // g.chunk_tokens * g.chunk_tokens
     reqs = [Request(prompt, matched, t, "host") for t in tables]
-    return Workload("llama8b", g, 20000, reqs)
+    name = "llama8b" if (requests, num_blocks) == (16, 20000) else f"llama8b_r{requests}_nb{num_blocks}"
+    return Workload(name, g, num_blocks, reqs)
 
 
 def sweep(ratio: float, requests: int = 32, prompt: int = 8192) -> Workload:

@@ -25,7 +25,7 @@ def test_library_exports_every_declared_function():
     for n in names:
         assert hasattr(lib, n), n
     assert set(names) == set(kvs.EXPORTED)
-    assert kvs.kvs_version() == 10000
+    assert kvs.kvs_version() == 10100
 
 
 def test_struct_layouts_match_header():
@@ -33,7 +33,7 @@ def test_struct_layouts_match_header():
     assert ctypes.sizeof(kvs.kvs_chunk) == 16
     assert ctypes.sizeof(kvs.kvs_request) == 40
     assert ctypes.sizeof(kvs.kvs_paged_cache) == 16
-    assert ctypes.sizeof(kvs.kvs_bw_report) == 5 * 8 + 6 * 8 + 4 * 4 + 8
+    assert ctypes.sizeof(kvs.kvs_bw_report) == 5 * 8 + 6 * 8 + 6 * 4 + 8
 
 
 FAKE = 0x10000   # never dereferenced: every case below fails validation first
