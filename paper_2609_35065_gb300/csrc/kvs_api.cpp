@@ -7,8 +7,8 @@
 // pinned slot copied on the caller's stream), then one kernel per source class
 // moves the bytes:
 //   device-resident chunks  -> LDG or TMA kernel, HBM to HBM;
-//   host-resident chunks    -> HOSTLINK: the LDG kernel loads/stores host memory
-//                              over the host link directly, or
+//   host-resident chunks    -> HOSTLINK: a double-buffered vector kernel loads/stores
+//                              host memory over the host link directly, or
 //                              HBMCOPY: the copy engine moves whole chunks
 //                              through a ring of HBM staging slots and the
 //                              device kernel scatters/gathers from there.
@@ -399,9 +399,14 @@ Job make_job(DevState& st, const kvs_geometry* g, const kvs_paged_cache* cache, 
     return j;
 }
 
+// Internal flavour: the double-buffered kernel used for host-resident chunks.
+constexpr int kKernelLink = 100;
+
 int launch_kernel(const Job& j, int flavour, int vec, int grid, cudaStream_t s) {
     if (j.num_pieces == 0) return KVS_OK;
-    cudaError_t e = (flavour == KVS_KERNEL_TMA) ? launch_tma(j, grid, s) : launch_ldg(j, vec, grid, s);
+    cudaError_t e = (flavour == KVS_KERNEL_TMA) ? launch_tma(j, grid, s)
+                  : (flavour == kKernelLink && vec == 16) ? launch_link(j, grid, s)
+                  : launch_ldg(j, vec, grid, s);
     if (e != cudaSuccess) return fail(KVS_ERR_CUDA, "kernel launch failed: %s", cudaGetErrorString(e));
     ++g_launches;
     return KVS_OK;
@@ -564,7 +569,7 @@ int copy_call(const kvs_geometry* g, const kvs_paged_cache* cache, const kvs_req
             rc = run_hbmcopy(st, g, cache, pl, u, mode, flavour, grid, s, host_addr);
         } else {
             rc = launch_kernel(make_job(st, g, cache, pl, u, pl.num_device, pl.num_host, mode),
-                               KVS_KERNEL_LDG, vec, host_grid, s);
+                               kKernelLink, vec, host_grid, s);
         }
         if (rc) return rc;
     }
@@ -689,18 +694,19 @@ int query_bw(DevState& st, kvs_bw_report* out, cudaStream_t s, int64_t probe_byt
     // Smallest host-link grid within 0.5% of the best: a grid that fills every SM
     // buys nothing once the link is saturated and starves concurrent kernels.
     {
-        const int full = st.sms * ldg_ctas_per_sm();
-        const int cand[] = {16, 24, 32, 48, 64, 96, 128, full};
-        double gb[2][8] = {};
+        const int full = st.sms * link_ctas_per_sm();
+        const int cand[] = {8, 12, 16, 24, 32, 48, 64, 96, 128, full};
+        constexpr int ncand = 10;
+        double gb[2][ncand] = {};
         for (int dir = 0; dir < 2; ++dir) {
             double best = 0;
-            for (int k = 0; k < 8; ++k) {
+            for (int k = 0; k < ncand; ++k) {
                 rc = probe_call(&rh, dir == 0, KVS_F_FORCE_HOSTLINK | KVS_F_MAX_CTAS(cand[k]), &gb[dir][k]);
                 if (rc) { cleanup(); return rc; }
                 best = std::max(best, gb[dir][k]);
             }
             int pick = 0;
-            for (int k = 0; k < 8; ++k)
+            for (int k = 0; k < ncand; ++k)
                 if (gb[dir][k] >= 0.995 * best) { pick = cand[k]; break; }
             if (pick >= full) pick = 0;
             if (dir == 0) rep.hostlink_ctas = pick; else rep.store_ctas = pick;

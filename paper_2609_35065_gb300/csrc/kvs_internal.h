@@ -48,6 +48,8 @@ constexpr uint32_t kPieceBytes = 32768;
 // Launchers (kvs_kernels.cu).  `grid` <= 0 means "fill the GPU".
 cudaError_t launch_ldg(const Job& job, int vec_bytes, int grid, cudaStream_t s);
 cudaError_t launch_tma(const Job& job, int grid, cudaStream_t s);
+// Double-buffered 16-byte flavour for host-resident chunks (retrieve or store).
+cudaError_t launch_link(const Job& job, int grid, cudaStream_t s);
 // Contiguous copy of `bytes` (multiple of 16, 16-byte aligned) for bandwidth probes.
 cudaError_t launch_flat_copy(void* dst, const void* src, uint64_t bytes, int grid, cudaStream_t s);
 // One CTA waits (bounded by limit_ns) on an mbarrier phase that nothing
@@ -57,6 +59,7 @@ cudaError_t launch_stall(int32_t* err, uint64_t limit_ns, cudaStream_t s);
 void set_last_error(const char* msg);
 // CTAs per SM the flavour runs with (occupancy); used to size persistent grids.
 int ldg_ctas_per_sm();
+int link_ctas_per_sm();
 int tma_ctas_per_sm();
 
 }  // namespace kvs

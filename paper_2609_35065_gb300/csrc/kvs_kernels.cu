@@ -9,6 +9,9 @@
 //    16-byte vector loads (non-coherent, no L1 allocation) issued ahead of
 //    16-byte streaming stores; persistent grid, grid-stride over pieces.
 //    Works for device and mapped-host sources and destinations.
+//  * LINK: the LDG scheme double-buffered in registers (the next piece's loads
+//    are issued before the current piece is stored), for host-resident
+//    chunks whose loads/stores cross the long-latency host link.
 //  * TMA: one thread per CTA drives a ring of shared-memory stages with 1-D
 //    bulk async copies (cp.async.bulk global->shared completing on an
 //    mbarrier, then shared->global bulk stores); every wait is bounded by the
@@ -181,6 +184,59 @@ __global__ void __launch_bounds__(kLdgThreads) kvs_ldg_kernel(const Decoder dc, 
             if (!equal_piece<V, kLdgUnroll>(pc.chunk_addr, pc.plane_addr, pc.len))
                 atomicCAS(j.err, 0, KVS_ERR_ALIAS);
         }
+    }
+}
+
+// Host-link flavour: each thread keeps two pieces' worth of 16-byte vectors in
+// registers, so the loads of the next piece are in flight while the current
+// one is stored.  A CTA then always has 32-64 KiB outstanding over the
+// long-latency host link, and a small grid saturates it.
+__device__ __forceinline__ bool next_piece_ldg(const Decoder& dc, uint32_t num_pieces, uint32_t& q, Piece& pc) {
+    while (q < num_pieces) {
+        const uint32_t cur = q;
+        q += gridDim.x;
+        if (decode_piece(dc, cur, pc)) return true;
+    }
+    return false;
+}
+
+__device__ __forceinline__ void load_piece16(uint64_t src, uint32_t len, uint4 (&r)[kLdgUnroll]) {
+    const uint4* s = reinterpret_cast<const uint4*>(src);
+    const uint32_t n = len / 16;
+#pragma unroll
+    for (int u = 0; u < kLdgUnroll; ++u) {
+        const uint32_t k = threadIdx.x + u * kLdgThreads;
+        if (k < n) r[u] = ld_stream<16>(s + k);
+    }
+}
+
+__device__ __forceinline__ void store_piece16(uint64_t dst, uint32_t len, const uint4 (&r)[kLdgUnroll]) {
+    uint4* d = reinterpret_cast<uint4*>(dst);
+    const uint32_t n = len / 16;
+#pragma unroll
+    for (int u = 0; u < kLdgUnroll; ++u) {
+        const uint32_t k = threadIdx.x + u * kLdgThreads;
+        if (k < n) st_stream<16>(d + k, r[u]);
+    }
+}
+
+template <int MODE>
+__global__ void __launch_bounds__(kLdgThreads) kvs_link_kernel(const Decoder dc, uint32_t num_pieces) {
+    static_assert(kPieceBytes == kLdgUnroll * kLdgThreads * 16, "one piece per register set");
+    constexpr bool to_plane = (MODE == MODE_RETRIEVE);
+    uint4 ra[kLdgUnroll], rb[kLdgUnroll];
+    Piece pa, pb;
+    uint32_t q = blockIdx.x;
+    bool ha = next_piece_ldg(dc, num_pieces, q, pa);
+    if (ha) load_piece16(to_plane ? pa.chunk_addr : pa.plane_addr, pa.len, ra);
+    while (ha) {
+        const bool hb = next_piece_ldg(dc, num_pieces, q, pb);
+        if (hb) load_piece16(to_plane ? pb.chunk_addr : pb.plane_addr, pb.len, rb);
+        store_piece16(to_plane ? pa.plane_addr : pa.chunk_addr, pa.len, ra);
+        if (!hb) break;
+        ha = next_piece_ldg(dc, num_pieces, q, pa);
+        if (ha) load_piece16(to_plane ? pa.chunk_addr : pa.plane_addr, pa.len, ra);
+        store_piece16(to_plane ? pb.plane_addr : pb.chunk_addr, pb.len, rb);
     }
 }
 
@@ -375,6 +431,27 @@ cudaError_t launch_ldg_v(const Job& job, int grid, cudaStream_t s) {
 }
 
 }  // namespace
+
+int link_ctas_per_sm() {
+    static int n = 0;
+    if (n == 0) {
+        cudaOccupancyMaxActiveBlocksPerMultiprocessor(&n, kvs_link_kernel<MODE_RETRIEVE>, kLdgThreads, 0);
+        if (n <= 0) n = 1;
+    }
+    return n;
+}
+
+cudaError_t launch_link(const Job& job, int grid, cudaStream_t s) {
+    if (job.num_pieces == 0) return cudaSuccess;
+    grid = clamp_grid(grid, link_ctas_per_sm(), job.num_pieces);
+    const Decoder dc = make_decoder(job);
+    const uint32_t n = (uint32_t)job.num_pieces;
+    if (job.mode == MODE_RETRIEVE)
+        kvs_link_kernel<MODE_RETRIEVE><<<grid, kLdgThreads, 0, s>>>(dc, n);
+    else
+        kvs_link_kernel<MODE_STORE><<<grid, kLdgThreads, 0, s>>>(dc, n);
+    return cudaGetLastError();
+}
 
 int ldg_ctas_per_sm() {
     static int n = 0;
