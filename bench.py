@@ -364,7 +364,7 @@ def run_ours(args):
     call_ms = statistics.mean(per_call_ms)
     value = whole_job_rate(payload, K, world, total_ms) / 1e9
     tokens_per_s = whole_job_rate(tokens, K, world, total_ms)
-    kernel_name = "kvs_ldg_kernel" if host_variant == 1 else "hbmcopy_pipeline"
+    kernel_name = "kvs_link_kernel" if host_variant == 1 else "hbmcopy_pipeline"
 
     # e2e: the public API from host arguments, result status read back every step
     e2e_steps = max(3, min(K, 20))
@@ -478,7 +478,7 @@ def run_ours(args):
         peak = payload / ideal_s / 1e9
         roofline = {"bound": "host_link+hbm", "achieved": round(achieved, 2), "peak": round(peak, 2),
                     "unit": "GB/s", "frac": round(achieved / peak, 4), "traffic": None,
-                    "kernel": "kvs_ldg_kernel (host) + device-class kernel on a second stream",
+                    "kernel": "kvs_link_kernel (host) + device-class kernel on a second stream",
                     "peak_source": "payload / max(host bytes / in-run host-link peak, "
                                    "2 x device bytes / MEASURED_PEAKS hbm_gbs)",
                     "bytes_counted": f"host {mv['host']} over the link, device {mv['device']} read+written in HBM"}

@@ -171,9 +171,9 @@ typedef struct kvs_bw_report {
     int32_t chosen_store_host;     /* KVS_VARIANT_* used for host chunks by kvs_store      */
     int32_t chosen_kernel_device;  /* KVS_KERNEL_* used for device-resident chunks         */
     int32_t num_sms;
-    int32_t hostlink_ctas;         /* CTAs given to host-link retrieval kernels (0 = all): the
-                                      smallest probed grid within 0.5% of the best rate, so
-                                      that kernels on other streams keep the remaining SMs */
+    int32_t hostlink_ctas;         /* CTAs given to host-link retrieval kernels (0 = all):
+                                      4 x the smallest probed grid within 0.5% of the best
+                                      rate, so that kernels on other streams keep most SMs */
     int32_t store_ctas;            /* the same for host-link store kernels                 */
     int64_t probe_bytes;           /* bytes moved per probe                                */
 } kvs_bw_report;

@@ -197,23 +197,41 @@ def _geometry(g) -> kvs_geometry:
     return kvs_geometry(*g)
 
 
+# numpy mirrors of kvs_chunk / kvs_request: one vectorised fill per call
+_CHUNK_DT = np.dtype([("base", "<u8"), ("num_tokens", "<i4"), ("residency", "<i4")])
+_REQ_DT = np.dtype([("first_token", "<i8"), ("num_tokens", "<i8"), ("chunks", "<u8"),
+                    ("num_chunks", "<i4"), ("block_table_len", "<i4"), ("block_table", "<u8")])
+assert _CHUNK_DT.itemsize == ctypes.sizeof(kvs_chunk) and _REQ_DT.itemsize == ctypes.sizeof(kvs_request)
+
+
 class _Marshalled:
-    """Keeps every ctypes array alive for the duration of one C call."""
+    """The C call's argument arrays (kept alive for the duration of one call)."""
 
     def __init__(self, planes, num_blocks, requests):
-        self.plane_arr = (ctypes.c_void_p * max(1, len(planes)))(*[_addr(p) for p in planes])
-        self.cache = kvs_paged_cache(ctypes.cast(self.plane_arr, ctypes.POINTER(ctypes.c_void_p)), int(num_blocks))
-        self.keep = []
-        self.reqs = (kvs_request * max(1, len(requests)))()
-        for k, r in enumerate(requests):
-            chunks = (kvs_chunk * max(1, len(r.chunks)))(
-                *[kvs_chunk(_addr(c.base), int(c.num_tokens), int(c.residency)) for c in r.chunks])
-            bt = np.ascontiguousarray(r.block_table, dtype=np.int32)
-            self.keep += [chunks, bt]
-            ntok = sum(int(c.num_tokens) for c in r.chunks) if r.num_tokens is None else int(r.num_tokens)
-            self.reqs[k] = kvs_request(int(r.first_token), ntok,
-                                       ctypes.cast(chunks, ctypes.POINTER(kvs_chunk)), len(r.chunks),
-                                       int(bt.size), bt.ctypes.data_as(ctypes.POINTER(ctypes.c_int32)))
+        self.planes = np.array([_addr(p) for p in planes] or [0], dtype=np.uint64)
+        self.cache = kvs_paged_cache(ctypes.cast(int(self.planes.ctypes.data), ctypes.POINTER(ctypes.c_void_p)),
+                                     int(num_blocks))
+        counts = [len(r.chunks) for r in requests]
+        chunks = np.zeros(max(1, sum(counts)), dtype=_CHUNK_DT)
+        flat = [c for r in requests for c in r.chunks]
+        if flat:
+            chunks["base"] = [_addr(c.base) for c in flat]
+            chunks["num_tokens"] = [c.num_tokens for c in flat]
+            chunks["residency"] = [c.residency for c in flat]
+        self.chunks = chunks
+        self.tables = [np.ascontiguousarray(r.block_table, dtype=np.int32) for r in requests]
+        reqs = np.zeros(max(1, len(requests)), dtype=_REQ_DT)
+        if requests:
+            starts = np.concatenate([[0], np.cumsum(counts)[:-1]]).astype(np.uint64)
+            reqs["first_token"] = [r.first_token for r in requests]
+            reqs["num_tokens"] = [sum(c.num_tokens for c in r.chunks) if r.num_tokens is None else r.num_tokens
+                                  for r in requests]
+            reqs["chunks"] = np.uint64(chunks.ctypes.data) + starts * np.uint64(_CHUNK_DT.itemsize)
+            reqs["num_chunks"] = counts
+            reqs["block_table_len"] = [t.size for t in self.tables]
+            reqs["block_table"] = [t.ctypes.data for t in self.tables]
+        self.reqs_np = reqs
+        self.reqs = ctypes.cast(int(reqs.ctypes.data), ctypes.POINTER(kvs_request))
         self.n = len(requests)
 
 
