@@ -279,7 +279,7 @@ int fill_plan(DevState& st, const kvs_geometry* g, const kvs_paged_cache* cache,
             }
             pl.entries[e].chunk = addr;
             pl.entries[e].n_tok = c.num_tokens;
-            pl.entries[e].blk_off = (int32_t)((uint64_t)e * pl.bpc);
+            pl.entries[e].pad = 0;
             pl.entry_bytes[e] = (uint64_t)P * c.num_tokens * pl.row_bytes;
             pl.addr_or |= addr;
             for (int32_t i = 0; i * B < c.num_tokens; ++i) {
@@ -388,6 +388,7 @@ Job make_job(DevState& st, const kvs_geometry* g, const kvs_paged_cache* cache, 
     j.row_bytes = pl.row_bytes;
     j.num_blocks = cache->num_blocks;
     j.num_entries = num_entries;
+    j.entry_base = first_entry;
     j.num_planes = (uint32_t)pl.planes.size();
     j.blocks_per_chunk = pl.bpc;
     j.piece_bytes = kPieceBytes;

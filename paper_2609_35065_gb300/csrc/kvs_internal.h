@@ -8,10 +8,12 @@
 namespace kvs {
 
 // One (request, chunk) pair of a call.  The chunk buffer is [L][2][n_tok][H][D].
+// Entry k's blocks are Job::blocks[k * blocks_per_chunk ...], so a kernel can
+// load a block id without waiting for the entry itself.
 struct Entry {
     uint64_t chunk;     // device-visible address of the chunk buffer
     int32_t  n_tok;     // tokens held by the chunk (its token stride)
-    int32_t  blk_off;   // index of the chunk's first block in Job::blocks
+    int32_t  pad;
 };
 static_assert(sizeof(Entry) == 16, "Entry is uploaded as raw bytes");
 
@@ -27,13 +29,15 @@ enum Mode : int32_t {
 // Run index g = (entry * num_planes + p) * blocks_per_chunk + i.
 struct Job {
     const Entry*    entries;
-    const int32_t*  blocks;          // physical block of (entry, i); < 0 means "skip"
+    const int32_t*  blocks;          // physical block of (entry k, i) at k * blocks_per_chunk + i;
+                                     // < 0 means "skip"
     const uint64_t* planes;          // 2L plane base addresses
     int32_t*        err;             // device error word (first error wins)
     uint64_t        row_bytes;       // R = H * D * e
     uint64_t        num_pieces;      // num_entries * num_planes * blocks_per_chunk * pieces_per_run
     int64_t         num_blocks;      // NB, for the device-side bounds check
     uint32_t        num_entries;
+    uint32_t        entry_base;      // index of entries[0] among all entries of the call
     uint32_t        num_planes;
     uint32_t        blocks_per_chunk;
     uint32_t        pieces_per_run;

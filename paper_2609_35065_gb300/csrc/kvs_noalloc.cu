@@ -193,7 +193,7 @@ int retrieve_noalloc(const kvs_geometry* g, const kvs_paged_cache* cache, const 
             const kvs_chunk& c = q.chunks[j];
             entries[e].chunk = (uint64_t)c.base;
             entries[e].n_tok = c.num_tokens;
-            entries[e].blk_off = (int32_t)(e * bpc);
+            entries[e].pad = 0;
             for (uint32_t i = 0; i < bpc; ++i) {
                 const uint32_t ref = e * bpc + i;
                 blocks[ref] = -1;
@@ -249,6 +249,7 @@ int retrieve_noalloc(const kvs_geometry* g, const kvs_paged_cache* cache, const 
     j.row_bytes = R;
     j.num_blocks = cache->num_blocks;
     j.num_entries = e;
+    j.entry_base = 0;
     j.num_planes = (uint32_t)P;
     j.blocks_per_chunk = bpc;
     j.piece_bytes = kPieceBytes;
