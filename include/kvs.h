@@ -157,6 +157,31 @@ int kvs_store(const kvs_geometry* geom, const kvs_paged_cache* cache,
               const kvs_request* requests, int32_t num_requests,
               void* cuda_stream, uint32_t flags);
 
+/*
+ * Layer-wise retrieval.  The paper's time-to-use ends when retrieval begins,
+ * not when the model consumes the KV (Sec. 3.1): the model can start on the
+ * first layers while later layers are still in flight.  This call does the
+ * same copy as kvs_retrieve, planned and uploaded once, as ceil(L /
+ * layers_per_step) launch groups in layer order on cuda_stream; after group k
+ * (layers [k * layers_per_step, (k + 1) * layers_per_step)) is enqueued,
+ * layer_events[k] is recorded on cuda_stream, so another stream can
+ * cudaStreamWaitEvent on it and use those layers while later groups copy.
+ * layer_events may be NULL, and so may any of its entries; the events are the
+ * caller's (cudaEvent_t cast to void*).  Host-resident chunks always take the
+ * host-link kernel here (KVS_F_FORCE_HBMCOPY returns KVS_ERR_UNSUPPORTED).
+ */
+int kvs_retrieve_layers(const kvs_geometry* geom, const kvs_paged_cache* cache,
+                        const kvs_request* requests, int32_t num_requests,
+                        int32_t layers_per_step, void* const* layer_events,
+                        void* cuda_stream, uint32_t flags);
+
+/* Layer-wise store-back: kvs_store in layer groups, recording layer_events[k]
+ * after group k (for storing KV while later layers are still being computed). */
+int kvs_store_layers(const kvs_geometry* geom, const kvs_paged_cache* cache,
+                     const kvs_request* requests, int32_t num_requests,
+                     int32_t layers_per_step, void* const* layer_events,
+                     void* cuda_stream, uint32_t flags);
+
 /* Bandwidths measured by kvs_query_bw, in GB/s (1e9 bytes per second). */
 typedef struct kvs_bw_report {
     double  hbm_copy_gbs;          /* device->device copy kernel, read + write bytes      */
@@ -252,7 +277,7 @@ int kvs_retrieve_noalloc(const kvs_geometry* geom, const kvs_paged_cache* cache,
 
 /* ABI version of this header: major * 10000 + minor * 100 + patch. */
 int kvs_version(void);
-#define KVS_VERSION 10100
+#define KVS_VERSION 10200
 
 #ifdef __cplusplus
 }

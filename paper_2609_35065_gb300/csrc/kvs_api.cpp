@@ -379,7 +379,8 @@ int upload(DevState& st, const Plan& pl, cudaStream_t s, Uploaded& u) {
 }
 
 Job make_job(DevState& st, const kvs_geometry* g, const kvs_paged_cache* cache, const Plan& pl,
-             const Uploaded& u, uint32_t first_entry, uint32_t num_entries, Mode mode) {
+             const Uploaded& u, uint32_t first_entry, uint32_t num_entries, Mode mode,
+             uint32_t plane_begin = 0, uint32_t plane_count = 0) {
     Job j{};
     j.entries = u.entries + first_entry;
     j.blocks = u.blocks;
@@ -389,7 +390,8 @@ Job make_job(DevState& st, const kvs_geometry* g, const kvs_paged_cache* cache, 
     j.num_blocks = cache->num_blocks;
     j.num_entries = num_entries;
     j.entry_base = first_entry;
-    j.num_planes = (uint32_t)pl.planes.size();
+    j.plane_begin = plane_begin;
+    j.num_planes = plane_count ? plane_count : (uint32_t)pl.planes.size() - plane_begin;
     j.blocks_per_chunk = pl.bpc;
     j.piece_bytes = kPieceBytes;
     j.block_size = (uint32_t)g->block_size;
@@ -515,21 +517,37 @@ int read_error_word(DevState& st, cudaStream_t s) {
     return KVS_OK;
 }
 
+// layers_per_step > 0: layer-wise copy, one launch group per `layers_per_step`
+// layers, each followed by a record of layer_events[group] (if given) on the
+// caller's stream.
 int copy_call(const kvs_geometry* g, const kvs_paged_cache* cache, const kvs_request* reqs,
-              int32_t nreq, void* stream, uint32_t flags, bool retrieve) {
+              int32_t nreq, void* stream, uint32_t flags, bool retrieve,
+              int32_t layers_per_step = 0, void* const* layer_events = nullptr) {
     const bool f_host = flags & KVS_F_FORCE_HOSTLINK, f_hbm = flags & KVS_F_FORCE_HBMCOPY;
     const bool f_ldg = flags & KVS_F_FORCE_LDG, f_tma = flags & KVS_F_FORCE_TMA;
     if ((f_host && f_hbm) || (f_ldg && f_tma))
         return fail(KVS_ERR_INVALID_ARG, "conflicting FORCE flags");
+    if (layers_per_step < 0) return fail(KVS_ERR_INVALID_ARG, "layers_per_step must be positive");
+    if (layers_per_step > 0 && f_hbm)
+        return fail(KVS_ERR_UNSUPPORTED, "layer-wise copies move host chunks over the host link only");
     Plan pl;
     int rc = validate_call(g, cache, reqs, nreq, pl);
     if (rc) return rc;
-    if (pl.num_device + pl.num_host == 0) return KVS_OK;
+    const int L = g->num_layers;
+    const int lps = layers_per_step > 0 ? std::min(layers_per_step, L) : L;
+    const int groups = (L + lps - 1) / lps;
+    cudaStream_t s = (cudaStream_t)stream;
+    if (pl.num_device + pl.num_host == 0) {
+        // nothing to copy: the layer events still mark "ready" in stream order
+        if (layers_per_step > 0 && layer_events)
+            for (int k = 0; k < groups; ++k)
+                if (layer_events[k]) KVS_CUDA(cudaEventRecord((cudaEvent_t)layer_events[k], s));
+        return KVS_OK;
+    }
     DevState* stp = nullptr;
     rc = get_state(&stp);
     if (rc) return rc;
     DevState& st = *stp;
-    cudaStream_t s = (cudaStream_t)stream;
     rc = fill_plan(st, g, cache, reqs, nreq, retrieve, flags, pl);
     if (rc) return rc;
     const int grid = (int)KVS_F_GET_MAX_CTAS(flags);
@@ -539,10 +557,10 @@ int copy_call(const kvs_geometry* g, const kvs_paged_cache* cache, const kvs_req
         if (f_tma) return fail(KVS_ERR_UNSUPPORTED, "TMA needs 16-byte aligned chunks, planes and rows");
         flavour = KVS_KERNEL_LDG;
     }
-    const int host_variant = f_host ? KVS_VARIANT_HOSTLINK : f_hbm ? KVS_VARIANT_HBMCOPY
-                                                                    : (retrieve ? st.retrieve_host : st.store_host);
+    int host_variant = f_host ? KVS_VARIANT_HOSTLINK : f_hbm ? KVS_VARIANT_HBMCOPY
+                                                            : (retrieve ? st.retrieve_host : st.store_host);
+    if (layers_per_step > 0) host_variant = KVS_VARIANT_HOSTLINK;
     const Mode mode = retrieve ? MODE_RETRIEVE : MODE_STORE;
-
     const int host_grid = grid ? grid : (retrieve ? st.hostlink_ctas : st.store_ctas);
 
     Uploaded u;
@@ -551,30 +569,36 @@ int copy_call(const kvs_geometry* g, const kvs_paged_cache* cache, const kvs_req
     // With both classes present, the HBM-bound device part runs on the aux
     // stream while the link-bound host part runs on the caller's stream.
     const bool fork = pl.num_device && pl.num_host;
-    if (pl.num_device) {
-        cudaStream_t ds = s;
-        if (fork) {
-            KVS_CUDA(cudaEventRecord(st.ev_aux_fork, s));
-            KVS_CUDA(cudaStreamWaitEvent(st.aux_stream, st.ev_aux_fork, 0));
-            ds = st.aux_stream;
+    for (int k = 0; k < groups; ++k) {
+        const uint32_t p0 = (uint32_t)(2 * k * lps);
+        const uint32_t np = (uint32_t)(2 * (std::min(L, (k + 1) * lps) - k * lps));
+        if (pl.num_device) {
+            cudaStream_t ds = s;
+            if (fork) {
+                KVS_CUDA(cudaEventRecord(st.ev_aux_fork, s));
+                KVS_CUDA(cudaStreamWaitEvent(st.aux_stream, st.ev_aux_fork, 0));
+                ds = st.aux_stream;
+            }
+            rc = launch_kernel(make_job(st, g, cache, pl, u, 0, pl.num_device, mode, p0, np), flavour, vec, grid, ds);
+            if (rc) return rc;
+            if (fork) KVS_CUDA(cudaEventRecord(st.ev_aux_join, st.aux_stream));
         }
-        rc = launch_kernel(make_job(st, g, cache, pl, u, 0, pl.num_device, mode), flavour, vec, grid, ds);
-        if (rc) return rc;
-        if (fork) KVS_CUDA(cudaEventRecord(st.ev_aux_join, st.aux_stream));
-    }
-    if (pl.num_host) {
-        if (host_variant == KVS_VARIANT_HBMCOPY) {
-            std::vector<const void*> host_addr(pl.num_host);
-            for (uint32_t e = pl.num_device; e < pl.entries.size(); ++e)
-                host_addr[e - pl.num_device] = (const void*)pl.entries[e].chunk;
-            rc = run_hbmcopy(st, g, cache, pl, u, mode, flavour, grid, s, host_addr);
-        } else {
-            rc = launch_kernel(make_job(st, g, cache, pl, u, pl.num_device, pl.num_host, mode),
-                               kKernelLink, vec, host_grid, s);
+        if (pl.num_host) {
+            if (host_variant == KVS_VARIANT_HBMCOPY) {
+                std::vector<const void*> host_addr(pl.num_host);
+                for (uint32_t e = pl.num_device; e < pl.entries.size(); ++e)
+                    host_addr[e - pl.num_device] = (const void*)pl.entries[e].chunk;
+                rc = run_hbmcopy(st, g, cache, pl, u, mode, flavour, grid, s, host_addr);
+            } else {
+                rc = launch_kernel(make_job(st, g, cache, pl, u, pl.num_device, pl.num_host, mode, p0, np),
+                                   kKernelLink, vec, host_grid, s);
+            }
+            if (rc) return rc;
         }
-        if (rc) return rc;
+        if (fork) KVS_CUDA(cudaStreamWaitEvent(s, st.ev_aux_join, 0));
+        if (layers_per_step > 0 && layer_events && layer_events[k])
+            KVS_CUDA(cudaEventRecord((cudaEvent_t)layer_events[k], s));
     }
-    if (fork) KVS_CUDA(cudaStreamWaitEvent(s, st.ev_aux_join, 0));
     if (!pl.blocks_cmp.empty()) {
         Job j = make_job(st, g, cache, pl, u, 0, (uint32_t)pl.entries.size(), MODE_COMPARE);
         j.blocks = u.blocks_cmp;
@@ -755,6 +779,24 @@ int kvs_store(const kvs_geometry* geom, const kvs_paged_cache* cache, const kvs_
     std::lock_guard<std::mutex> lk(g_mu);
     t_error.clear();
     return copy_call(geom, cache, requests, num_requests, cuda_stream, flags, false);
+}
+
+int kvs_retrieve_layers(const kvs_geometry* geom, const kvs_paged_cache* cache, const kvs_request* requests,
+                        int32_t num_requests, int32_t layers_per_step, void* const* layer_events,
+                        void* cuda_stream, uint32_t flags) {
+    std::lock_guard<std::mutex> lk(g_mu);
+    t_error.clear();
+    if (layers_per_step <= 0) return fail(KVS_ERR_INVALID_ARG, "layers_per_step must be positive");
+    return copy_call(geom, cache, requests, num_requests, cuda_stream, flags, true, layers_per_step, layer_events);
+}
+
+int kvs_store_layers(const kvs_geometry* geom, const kvs_paged_cache* cache, const kvs_request* requests,
+                     int32_t num_requests, int32_t layers_per_step, void* const* layer_events,
+                     void* cuda_stream, uint32_t flags) {
+    std::lock_guard<std::mutex> lk(g_mu);
+    t_error.clear();
+    if (layers_per_step <= 0) return fail(KVS_ERR_INVALID_ARG, "layers_per_step must be positive");
+    return copy_call(geom, cache, requests, num_requests, cuda_stream, flags, false, layers_per_step, layer_events);
 }
 
 int kvs_query_bw(kvs_bw_report* out, void* cuda_stream, int64_t probe_bytes) {

@@ -38,7 +38,8 @@ struct Job {
     int64_t         num_blocks;      // NB, for the device-side bounds check
     uint32_t        num_entries;
     uint32_t        entry_base;      // index of entries[0] among all entries of the call
-    uint32_t        num_planes;
+    uint32_t        num_planes;      // planes copied by this launch ...
+    uint32_t        plane_begin;     // ... starting at this plane (2 * first layer)
     uint32_t        blocks_per_chunk;
     uint32_t        pieces_per_run;
     uint32_t        piece_bytes;     // multiple of 16

@@ -69,7 +69,7 @@ __device__ __forceinline__ bool decode_piece(const Decoder& dc, uint32_t q, Piec
     const uint32_t ep = fdiv(g, dc.bpc);
     const uint32_t i = g - ep * dc.bpc.d;
     const uint32_t e = fdiv(ep, dc.planes);
-    const uint32_t p = ep - e * dc.planes.d;
+    const uint32_t p = j.plane_begin + (ep - e * dc.planes.d);
     // The two descriptor loads are independent, so both are in flight at once.
     const int32_t blk = __ldg(j.blocks + (size_t)(j.entry_base + e) * j.blocks_per_chunk + i);
     const Entry en = j.entries[e];

@@ -251,6 +251,7 @@ int retrieve_noalloc(const kvs_geometry* g, const kvs_paged_cache* cache, const 
     j.num_entries = e;
     j.entry_base = 0;
     j.num_planes = (uint32_t)P;
+    j.plane_begin = 0;
     j.blocks_per_chunk = bpc;
     j.piece_bytes = kPieceBytes;
     j.block_size = (uint32_t)B;

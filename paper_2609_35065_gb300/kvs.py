@@ -55,7 +55,7 @@ KVS_KERNEL_TMA = 2
 
 EXPORTED = ("kvs_retrieve", "kvs_store", "kvs_query_bw", "kvs_get_choice", "kvs_check_errors",
             "kvs_last_error", "kvs_shutdown", "kvs_version", "kvs_selftest_wait_timeout",
-            "kvs_stat_launches", "kvs_retrieve_noalloc")
+            "kvs_stat_launches", "kvs_retrieve_noalloc", "kvs_retrieve_layers", "kvs_store_layers")
 KVS_NOALLOC_SCRATCH_BYTES = 1 << 20
 
 
@@ -130,6 +130,12 @@ def lib():
                 fn = getattr(L, name)
                 fn.argtypes = [ctypes.POINTER(kvs_geometry), ctypes.POINTER(kvs_paged_cache),
                                ctypes.POINTER(kvs_request), ctypes.c_int32, P, ctypes.c_uint32]
+                fn.restype = ctypes.c_int
+            for name in ("kvs_retrieve_layers", "kvs_store_layers"):
+                fn = getattr(L, name)
+                fn.argtypes = [ctypes.POINTER(kvs_geometry), ctypes.POINTER(kvs_paged_cache),
+                               ctypes.POINTER(kvs_request), ctypes.c_int32, ctypes.c_int32,
+                               ctypes.POINTER(ctypes.c_void_p), P, ctypes.c_uint32]
                 fn.restype = ctypes.c_int
             L.kvs_query_bw.argtypes = [ctypes.POINTER(kvs_bw_report), P, ctypes.c_int64]
             L.kvs_query_bw.restype = ctypes.c_int
@@ -257,6 +263,48 @@ def kvs_store(geom, planes, num_blocks, requests, stream=None, flags: int = 0) -
     m = _Marshalled(planes, num_blocks, requests)
     return _check(lib().kvs_store(ctypes.byref(g), ctypes.byref(m.cache), m.reqs, m.n,
                                   _stream(stream), ctypes.c_uint32(flags)))
+
+
+def _events(events, stream):
+    """cudaEvent_t handles of ``events``.  torch creates an event's handle at its first
+    record, so a fresh ``torch.cuda.Event`` is first recorded once on the current
+    stream; the library's record, made later in host order, is the one that waits see."""
+    if events is None:
+        return None, None
+    handles = []
+    for e in events:
+        if e is None:
+            handles.append(0)
+        elif hasattr(e, "cuda_event"):
+            if not int(e.cuda_event):
+                import torch
+                e.record(torch.cuda.current_stream())
+            handles.append(int(e.cuda_event))
+        else:
+            handles.append(int(e))
+    arr = (ctypes.c_void_p * max(1, len(handles)))(*handles)
+    return arr, ctypes.cast(arr, ctypes.POINTER(ctypes.c_void_p))
+
+
+def kvs_retrieve_layers(geom, planes, num_blocks, requests, layers_per_step, layer_events=None,
+                        stream=None, flags: int = 0) -> int:
+    """Layer-wise :func:`kvs_retrieve`: ``layer_events[k]`` (``torch.cuda.Event`` or raw
+    ``cudaEvent_t``) is recorded on ``stream`` after layer group k is enqueued."""
+    g = _geometry(geom)
+    m = _Marshalled(planes, num_blocks, requests)
+    keep, ev = _events(layer_events, stream)
+    return _check(lib().kvs_retrieve_layers(ctypes.byref(g), ctypes.byref(m.cache), m.reqs, m.n,
+                                            int(layers_per_step), ev, _stream(stream), ctypes.c_uint32(flags)))
+
+
+def kvs_store_layers(geom, planes, num_blocks, requests, layers_per_step, layer_events=None,
+                     stream=None, flags: int = 0) -> int:
+    """Layer-wise :func:`kvs_store`."""
+    g = _geometry(geom)
+    m = _Marshalled(planes, num_blocks, requests)
+    keep, ev = _events(layer_events, stream)
+    return _check(lib().kvs_store_layers(ctypes.byref(g), ctypes.byref(m.cache), m.reqs, m.n,
+                                         int(layers_per_step), ev, _stream(stream), ctypes.c_uint32(flags)))
 
 
 def kvs_query_bw(stream=None, probe_bytes: int = 0) -> dict:

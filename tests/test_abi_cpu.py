@@ -25,7 +25,7 @@ def test_library_exports_every_declared_function():
     for n in names:
         assert hasattr(lib, n), n
     assert set(names) == set(kvs.EXPORTED)
-    assert kvs.kvs_version() == 10100
+    assert kvs.kvs_version() == 10200
 
 
 def test_struct_layouts_match_header():
@@ -95,3 +95,17 @@ def test_call_too_large_is_rejected():
 def test_empty_call_needs_no_device():
     assert kvs.kvs_retrieve(G, [FAKE] * 4, 8, [], None, 0) == kvs.KVS_OK
     assert kvs.kvs_store(G, [FAKE] * 4, 8, [_req(tokens=(), table=())], None, 0) == kvs.KVS_OK
+
+
+@pytest.mark.parametrize("fn", [kvs.kvs_retrieve_layers, kvs.kvs_store_layers])
+def test_layerwise_argument_checks(fn):
+    with pytest.raises(kvs.KvsError) as ei:
+        fn(G, [FAKE] * 4, 8, [_req()], 0)
+    assert ei.value.code == kvs.KVS_ERR_INVALID_ARG
+    with pytest.raises(kvs.KvsError) as ei:
+        fn(G, [FAKE] * 4, 8, [_req()], 1, None, None, kvs.KVS_F_FORCE_HBMCOPY)
+    assert ei.value.code == kvs.KVS_ERR_UNSUPPORTED
+    with pytest.raises(kvs.KvsError) as ei:
+        fn(G, [FAKE] * 4, 8, [_req(table=(0, 1, 9, 3))], 1)
+    assert ei.value.code == kvs.KVS_ERR_BOUNDS
+    assert fn(G, [FAKE] * 4, 8, [], 1) == kvs.KVS_OK          # nothing to copy, no events given
