@@ -198,7 +198,8 @@ typedef struct kvs_bw_report {
     int32_t num_sms;
     int32_t hostlink_ctas;         /* CTAs given to host-link retrieval kernels (0 = all):
                                       4 x the smallest probed grid within 0.5% of the best
-                                      rate, so that kernels on other streams keep most SMs */
+                                      rate, so that kernels on other streams keep most SMs
+                                      (before any kvs_query_bw: one per 3 SMs)            */
     int32_t store_ctas;            /* the same for host-link store kernels                 */
     int64_t probe_bytes;           /* bytes moved per probe                                */
 } kvs_bw_report;

@@ -103,12 +103,9 @@ def allocate(w: synth.Workload, device: str = "cuda", store: bool = False,
     pin = torch.device(device).type == "cuda"
 
     dt = _DTYPES[g.elem_bytes]
-    sent = torch.tensor(synth.sentinel(g.elem_bytes), dtype=torch.int64)
-    if g.elem_bytes < 8:
-        sent = sent.to(torch.int64).numpy().astype(NP_DTYPES[g.elem_bytes]).view(
-            {1: np.uint8, 2: np.int16, 4: np.int32}[g.elem_bytes]).item()
-    else:
-        sent = int(np.array([synth.sentinel(8)], dtype=np.uint64).view(np.int64)[0])
+    # the sentinel's bit pattern as a value of the (signed) storage dtype
+    sent = int(np.array([synth.sentinel(g.elem_bytes)], dtype=NP_DTYPES[g.elem_bytes])
+               .view({1: np.uint8, 2: np.int16, 4: np.int32, 8: np.int64}[g.elem_bytes])[0])
     planes = None
     if with_planes:
         n = w.num_blocks * g.block_size * g.row_elems

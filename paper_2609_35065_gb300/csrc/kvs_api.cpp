@@ -115,7 +115,12 @@ int get_state(DevState** out) {
         KVS_CUDA(cudaStreamCreateWithFlags(&st.aux_stream, cudaStreamNonBlocking));
         KVS_CUDA(cudaEventCreateWithFlags(&st.ev_aux_fork, cudaEventDisableTiming));
         KVS_CUDA(cudaEventCreateWithFlags(&st.ev_aux_join, cudaEventDisableTiming));
+        // Until kvs_query_bw measures them, host-link kernels take a third of the
+        // SMs' worth of CTAs: enough to saturate the link, not the whole GPU.
+        st.hostlink_ctas = st.store_ctas = std::max(8, st.sms / 3);
         st.report.num_sms = st.sms;
+        st.report.hostlink_ctas = st.hostlink_ctas;
+        st.report.store_ctas = st.store_ctas;
         st.report.chosen_retrieve_host = st.retrieve_host;
         st.report.chosen_store_host = st.store_host;
         st.report.chosen_kernel_device = st.kernel_device;
