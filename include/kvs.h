@@ -276,9 +276,110 @@ int kvs_retrieve_noalloc(const kvs_geometry* geom, const kvs_paged_cache* cache,
                          const kvs_request* requests, int32_t num_requests,
                          void* cuda_stream, uint32_t flags);
 
+/* ======================================================================
+ * Fast tier: the objects retrieval reads from, and their protection.
+ *
+ * TempoKV's storage-side provider (Sec. 3.2, Sec. 4) keeps reusable KV
+ * objects in a fast tier shared by protected staging and ordinary caching:
+ *  - a protected-capacity budget below the tier's capacity counts protected
+ *    objects and reservations for outstanding staging, each shared object
+ *    once, without partitioning memory statically;
+ *  - committing a claim protects each object of its manifest, staging the
+ *    ones not resident (staging of one object is coalesced across claims);
+ *    a claim whose additional footprint does not fit the budget stays Planned;
+ *  - a claim is StageReady once every object is resident and protected, and
+ *    Transferring from the start of its GPU retrieval; protection ends when
+ *    that retrieval completes (Released), unprotected objects stay resident
+ *    as evictable cache entries (LRU);
+ *  - cancelling a committed claim keeps its protection until its outstanding
+ *    staging and GPU accesses end;
+ *  - the ordinary (demand) path reserves nothing and, once selected for a
+ *    claim, excludes its commitment;
+ *  - the protected-capacity cost is C = (integral of P(t) dt) / N (Sec. 5).
+ * One object = one KV chunk of object_bytes.  Every call takes the caller's
+ * clock `now` (seconds, non-decreasing) so that P(t) is integrated exactly.
+ * The tier is a host-side ledger; with arena != 0 it also owns a pinned,
+ * device-mapped host arena of capacity_objects slots that kvs_retrieve can
+ * read (the fast-tier stand-in).  Not thread-safe: one tier per thread.
+ * ====================================================================== */
+typedef struct kvs_tier kvs_tier;
+
+typedef struct kvs_tier_config {
+    int64_t capacity_objects;   /* slots in the fast tier                         */
+    int64_t budget_objects;     /* protected-capacity budget, < capacity_objects  */
+    int64_t object_bytes;       /* bytes of one object (one chunk)                */
+    int32_t arena;              /* 1: allocate the pinned arena, 0: ledger only   */
+    int32_t reserved;
+} kvs_tier_config;
+
+/* claim states */
+#define KVS_CLAIM_NONE         0
+#define KVS_CLAIM_PLANNED      1
+#define KVS_CLAIM_STAGING      2
+#define KVS_CLAIM_STAGE_READY  3
+#define KVS_CLAIM_TRANSFERRING 4
+#define KVS_CLAIM_RELEASED     5
+#define KVS_CLAIM_CANCELLED    6
+#define KVS_CLAIM_ORDINARY     7   /* ordinary retrieval selected (never protected) */
+
+typedef struct kvs_tier_object_info {
+    int64_t slot;               /* -1 when the object holds no slot               */
+    int32_t pins;               /* claims protecting it                           */
+    int32_t staging;            /* 1 while its staging I/O is outstanding         */
+    int32_t resident;           /* 1 once its bytes are in the slot               */
+    int32_t gpu_refs;           /* retrievals in progress that read it            */
+    uint64_t lru;               /* last-use stamp (logical clock)                 */
+} kvs_tier_object_info;
+
+typedef struct kvs_tier_stats {
+    int64_t resident, staging, protected_objects, free_slots, evictions;
+    int64_t staged_reads;       /* staging I/Os issued (coalesced ones count once) */
+    int64_t completed;          /* claims Released (N of the cost C)              */
+    double  protected_object_seconds;   /* integral of P(t) dt, in objects x s   */
+} kvs_tier_stats;
+
+int kvs_tier_create(const kvs_tier_config* cfg, kvs_tier** out);
+int kvs_tier_destroy(kvs_tier* tier);
+
+/* Commit `claim` (a new id, or a Planned one being retried) with the ordered
+ * manifest keys[0..n).  On KVS_OK the claim is Staging or StageReady and
+ * stage_keys[0..*n_stage) receive the objects whose staging I/O the caller
+ * must now perform (fill the slot, see kvs_tier_slot, then kvs_tier_staged);
+ * stage_keys needs room for n keys.  KVS_ERR_NOMEM: the footprint does not fit
+ * the budget (or no slot can be freed); the claim is Planned and nothing else
+ * changed.  KVS_ERR_INVALID_ARG: duplicate keys, a claim past Planned, or one
+ * on the ordinary path. */
+int kvs_tier_commit(kvs_tier* tier, uint64_t claim, const uint64_t* keys, int32_t n,
+                    double now, uint64_t* stage_keys, int32_t* n_stage);
+/* Staging I/O of `key` completed: the object is resident; claims waiting only
+ * on it become StageReady. */
+int kvs_tier_staged(kvs_tier* tier, uint64_t key, double now);
+/* Retrieval of a StageReady claim begins (Transferring); slots_out[i] gets the
+ * slot of keys[i] of its manifest. */
+int kvs_tier_begin_retrieval(kvs_tier* tier, uint64_t claim, double now, int64_t* slots_out);
+/* The claim's GPU retrieval completed: protection on its behalf ends (Released). */
+int kvs_tier_end_retrieval(kvs_tier* tier, uint64_t claim, double now);
+/* Cancel a claim: Planned ones at once; committed ones keep their protection
+ * until their outstanding staging and GPU accesses end. */
+int kvs_tier_cancel(kvs_tier* tier, uint64_t claim, double now);
+/* Select the ordinary (demand) path for a claim that is not committed: its
+ * objects are held for the retrieval without protection; stage_keys receive
+ * the non-resident ones to fetch on demand (into evictable slots).  Finish with
+ * kvs_tier_staged for each, then kvs_tier_begin_retrieval / end_retrieval. */
+int kvs_tier_ordinary(kvs_tier* tier, uint64_t claim, const uint64_t* keys, int32_t n,
+                      double now, uint64_t* stage_keys, int32_t* n_stage);
+
+int kvs_tier_claim_state(const kvs_tier* tier, uint64_t claim);          /* KVS_CLAIM_* */
+int kvs_tier_object(const kvs_tier* tier, uint64_t key, kvs_tier_object_info* out); /* KVS_ERR_BOUNDS if unknown */
+int kvs_tier_stats_get(kvs_tier* tier, double now, kvs_tier_stats* out);
+/* Host address of a slot in the arena (NULL without an arena or out of range);
+ * arena slots are pinned and device-mapped: pass them to kvs_retrieve as
+ * KVS_SRC_HOST_PINNED chunks. */
+void* kvs_tier_slot(const kvs_tier* tier, int64_t slot);
+
 /* ABI version of this header: major * 10000 + minor * 100 + patch. */
 int kvs_version(void);
-#define KVS_VERSION 10200
+#define KVS_VERSION 10300
 
 #ifdef __cplusplus
 }

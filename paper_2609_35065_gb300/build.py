@@ -17,7 +17,7 @@ CSRC = os.path.join(PKG, "csrc")
 INCLUDE = os.path.join(ROOT, "include")
 OUT_DIR = os.path.join(PKG, "_build")
 LIB = os.path.join(OUT_DIR, "libkvs.so")
-SOURCES = [os.path.join(CSRC, f) for f in ("kvs_kernels.cu", "kvs_api.cpp", "kvs_noalloc.cu")]
+SOURCES = [os.path.join(CSRC, f) for f in ("kvs_kernels.cu", "kvs_api.cpp", "kvs_noalloc.cu", "kvs_tier.cpp")]
 DEPS = SOURCES + [os.path.join(CSRC, "kvs_internal.h"), os.path.join(INCLUDE, "kvs.h")]
 ARCH = "-gencode=arch=compute_103a,code=sm_103a"
 
@@ -31,7 +31,7 @@ def nvcc() -> str:
 
 def command(out: str = LIB, extra: list[str] | None = None) -> list[str]:
     return [nvcc(), "-O3", "-lineinfo", "-std=c++17", ARCH, "-Xcompiler", "-fPIC,-O2,-Wall",
-            "-shared", "--threads", "3", "-I", INCLUDE, *SOURCES, "-o", out, *(extra or [])]
+            "-shared", "--threads", "4", "-I", INCLUDE, *SOURCES, "-o", out, *(extra or [])]
 
 
 def stale(out: str = LIB) -> bool:

@@ -55,7 +55,14 @@ KVS_KERNEL_TMA = 2
 
 EXPORTED = ("kvs_retrieve", "kvs_store", "kvs_query_bw", "kvs_get_choice", "kvs_check_errors",
             "kvs_last_error", "kvs_shutdown", "kvs_version", "kvs_selftest_wait_timeout",
-            "kvs_stat_launches", "kvs_retrieve_noalloc", "kvs_retrieve_layers", "kvs_store_layers")
+            "kvs_stat_launches", "kvs_retrieve_noalloc", "kvs_retrieve_layers", "kvs_store_layers",
+            "kvs_tier_create", "kvs_tier_destroy", "kvs_tier_commit", "kvs_tier_staged",
+            "kvs_tier_begin_retrieval", "kvs_tier_end_retrieval", "kvs_tier_cancel", "kvs_tier_ordinary",
+            "kvs_tier_claim_state", "kvs_tier_object", "kvs_tier_stats_get", "kvs_tier_slot")
+KVS_CLAIM_NONE, KVS_CLAIM_PLANNED, KVS_CLAIM_STAGING, KVS_CLAIM_STAGE_READY = 0, 1, 2, 3
+KVS_CLAIM_TRANSFERRING, KVS_CLAIM_RELEASED, KVS_CLAIM_CANCELLED, KVS_CLAIM_ORDINARY = 4, 5, 6, 7
+CLAIM_NAMES = {0: "None", 1: "Planned", 2: "Staging", 3: "StageReady", 4: "Transferring",
+               5: "Released", 6: "Cancelled", 7: "Ordinary"}
 KVS_NOALLOC_SCRATCH_BYTES = 1 << 20
 
 
@@ -104,6 +111,22 @@ class kvs_bw_report(ctypes.Structure):
         return out
 
 
+class kvs_tier_config(ctypes.Structure):
+    _fields_ = [("capacity_objects", ctypes.c_int64), ("budget_objects", ctypes.c_int64),
+                ("object_bytes", ctypes.c_int64), ("arena", ctypes.c_int32), ("reserved", ctypes.c_int32)]
+
+
+class kvs_tier_object_info(ctypes.Structure):
+    _fields_ = [("slot", ctypes.c_int64), ("pins", ctypes.c_int32), ("staging", ctypes.c_int32),
+                ("resident", ctypes.c_int32), ("gpu_refs", ctypes.c_int32), ("lru", ctypes.c_uint64)]
+
+
+class kvs_tier_stats(ctypes.Structure):
+    _fields_ = [("resident", ctypes.c_int64), ("staging", ctypes.c_int64), ("protected_objects", ctypes.c_int64),
+                ("free_slots", ctypes.c_int64), ("evictions", ctypes.c_int64), ("staged_reads", ctypes.c_int64),
+                ("completed", ctypes.c_int64), ("protected_object_seconds", ctypes.c_double)]
+
+
 # ---- library loading ------------------------------------------------------
 _lock = threading.Lock()
 _lib = None
@@ -137,6 +160,27 @@ def lib():
                                ctypes.POINTER(kvs_request), ctypes.c_int32, ctypes.c_int32,
                                ctypes.POINTER(ctypes.c_void_p), P, ctypes.c_uint32]
                 fn.restype = ctypes.c_int
+            U64P, I64P, I32P = (ctypes.POINTER(ctypes.c_uint64), ctypes.POINTER(ctypes.c_int64),
+                                ctypes.POINTER(ctypes.c_int32))
+            tier_sigs = {
+                "kvs_tier_create": [ctypes.POINTER(kvs_tier_config), ctypes.POINTER(P)],
+                "kvs_tier_destroy": [P],
+                "kvs_tier_commit": [P, ctypes.c_uint64, U64P, ctypes.c_int32, ctypes.c_double, U64P, I32P],
+                "kvs_tier_ordinary": [P, ctypes.c_uint64, U64P, ctypes.c_int32, ctypes.c_double, U64P, I32P],
+                "kvs_tier_staged": [P, ctypes.c_uint64, ctypes.c_double],
+                "kvs_tier_begin_retrieval": [P, ctypes.c_uint64, ctypes.c_double, I64P],
+                "kvs_tier_end_retrieval": [P, ctypes.c_uint64, ctypes.c_double],
+                "kvs_tier_cancel": [P, ctypes.c_uint64, ctypes.c_double],
+                "kvs_tier_claim_state": [P, ctypes.c_uint64],
+                "kvs_tier_object": [P, ctypes.c_uint64, ctypes.POINTER(kvs_tier_object_info)],
+                "kvs_tier_stats_get": [P, ctypes.c_double, ctypes.POINTER(kvs_tier_stats)],
+            }
+            for name, sig in tier_sigs.items():
+                fn = getattr(L, name)
+                fn.argtypes = sig
+                fn.restype = ctypes.c_int
+            L.kvs_tier_slot.argtypes = [P, ctypes.c_int64]
+            L.kvs_tier_slot.restype = ctypes.c_void_p
             L.kvs_query_bw.argtypes = [ctypes.POINTER(kvs_bw_report), P, ctypes.c_int64]
             L.kvs_query_bw.restype = ctypes.c_int
             L.kvs_get_choice.argtypes = [ctypes.POINTER(kvs_bw_report)]
@@ -352,3 +396,83 @@ def kvs_retrieve_noalloc(geom, planes, num_blocks, requests, stream=None, flags:
     m = _Marshalled(planes, num_blocks, requests)
     return _check(lib().kvs_retrieve_noalloc(ctypes.byref(g), ctypes.byref(m.cache), m.reqs, m.n,
                                              _stream(stream), ctypes.c_uint32(flags)))
+
+
+# ---- fast tier ------------------------------------------------------------
+def _u64(keys):
+    a = np.ascontiguousarray(np.asarray(keys, dtype=np.uint64))
+    return a, a.ctypes.data_as(ctypes.POINTER(ctypes.c_uint64))
+
+
+class Tier:
+    """The fast tier's ledger (and optional pinned arena): thin wrapper over kvs_tier_*.
+    Every method takes the caller's clock ``now`` in seconds."""
+
+    def __init__(self, capacity_objects: int, budget_objects: int, object_bytes: int, arena: bool = False):
+        cfg = kvs_tier_config(int(capacity_objects), int(budget_objects), int(object_bytes), int(bool(arena)), 0)
+        h = ctypes.c_void_p()
+        _check(lib().kvs_tier_create(ctypes.byref(cfg), ctypes.byref(h)))
+        self.handle = h
+        self.object_bytes = int(object_bytes)
+
+    def close(self):
+        if self.handle:
+            lib().kvs_tier_destroy(self.handle)
+            self.handle = None
+
+    def __del__(self):
+        try:
+            self.close()
+        except Exception:
+            pass
+
+    def _staging_call(self, fn, claim, keys, now):
+        ks, kp = _u64(keys)
+        out = np.zeros(max(1, ks.size), dtype=np.uint64)
+        n = ctypes.c_int32(0)
+        _check(fn(self.handle, int(claim), kp, int(ks.size), float(now),
+                  out.ctypes.data_as(ctypes.POINTER(ctypes.c_uint64)), ctypes.byref(n)))
+        return [int(x) for x in out[:n.value]]
+
+    def commit(self, claim, keys, now):
+        """kvs_tier_commit: returns the keys whose staging the caller must now perform."""
+        return self._staging_call(lib().kvs_tier_commit, claim, keys, now)
+
+    def ordinary(self, claim, keys, now):
+        """kvs_tier_ordinary: returns the keys to fetch on demand."""
+        return self._staging_call(lib().kvs_tier_ordinary, claim, keys, now)
+
+    def staged(self, key, now):
+        _check(lib().kvs_tier_staged(self.handle, int(key), float(now)))
+
+    def begin_retrieval(self, claim, now, n_keys):
+        slots = np.zeros(max(1, n_keys), dtype=np.int64)
+        _check(lib().kvs_tier_begin_retrieval(self.handle, int(claim), float(now),
+                                              slots.ctypes.data_as(ctypes.POINTER(ctypes.c_int64))))
+        return [int(x) for x in slots[:n_keys]]
+
+    def end_retrieval(self, claim, now):
+        _check(lib().kvs_tier_end_retrieval(self.handle, int(claim), float(now)))
+
+    def cancel(self, claim, now):
+        _check(lib().kvs_tier_cancel(self.handle, int(claim), float(now)))
+
+    def state(self, claim) -> int:
+        return int(lib().kvs_tier_claim_state(self.handle, int(claim)))
+
+    def object(self, key):
+        info = kvs_tier_object_info()
+        rc = lib().kvs_tier_object(self.handle, int(key), ctypes.byref(info))
+        if rc == KVS_ERR_BOUNDS:
+            return None
+        _check(rc)
+        return {"slot": info.slot, "pins": info.pins, "staging": info.staging, "resident": info.resident,
+                "gpu_refs": info.gpu_refs, "lru": info.lru}
+
+    def stats(self, now) -> dict:
+        st = kvs_tier_stats()
+        _check(lib().kvs_tier_stats_get(self.handle, float(now), ctypes.byref(st)))
+        return {name: getattr(st, name) for name, _ in st._fields_}
+
+    def slot_address(self, slot) -> int:
+        return int(lib().kvs_tier_slot(self.handle, int(slot)) or 0)
