@@ -51,6 +51,8 @@ def parse_args(argv=None):
     ap.add_argument("--overlap", action="store_true", help="llama70b: retrieval beside a bf16 GEMM loop")
     ap.add_argument("--layerwise", action="store_true",
                     help="llama8b: layer-wise retrieval pipelined with a per-layer prefill GEMM")
+    ap.add_argument("--tempokv", action="store_true",
+                    help="TempoKV control-plane model driven by the retrieval rate measured in this run")
     ap.add_argument("--side-priority", choices=["normal", "high"], default="high",
                     help="priority of the retrieval stream in --overlap runs")
     return ap.parse_args(argv)
@@ -706,8 +708,52 @@ def run_layerwise(args):
     return 0
 
 
+def run_tempokv(args):
+    """The control-plane model (12 synthetic documents, prefix ratios 50/75/100%,
+    100 GiB fast tier, 50 GiB protected budget, 11 GiB/s staging) with the
+    fast-tier -> GPU rate measured now by kvs_query_bw, and with the ~16.8 GB/s
+    effective rate implied by the paper's own H100 PCIe measurement."""
+    import time as _time
+
+    import numpy as np
+    from paper_2609_35065_gb300 import kvs, tempokv
+    measured = None
+    try:
+        import torch
+        if torch.cuda.is_available():
+            torch.cuda.set_device(0)
+            rep = kvs.kvs_query_bw(None, 1 << 30)
+            measured = max(rep["retrieve_gbs"])
+    except Exception:                                   # no GPU: the model alone
+        measured = None
+    rates = {"pcie_context_16.8": 16.8}
+    if measured:
+        rates["gb300_measured"] = round(measured, 2)
+    out = {}
+    t0 = _time.perf_counter()
+    for name, gbs in rates.items():
+        cal = tempokv.Calibration(retrieval_gbs=gbs)
+        for ratio in (0.5, 0.75, 1.0):
+            res = tempokv.simulate(tempokv.workload(ratio, cal=cal), cal)
+            out[f"{name}/ratio{int(ratio * 100)}"] = {
+                "p95_ttft_s": round(res.p95_ttft, 3), "throughput_tok_s": round(res.throughput_tok_s, 2),
+                "C_gib_s_per_req": round(res.cost_gib_s_per_req, 3), "blocked_commit_attempts": res.blocked_attempts,
+                "ordinary_retrievals": res.ordinary,
+                "mean_commit_lead_s": round(float(np.mean(res.commit_lead_s)), 3) if res.commit_lead_s else None}
+    line = {"metric": "TempoKV control-plane model: p95 TTFT, throughput and protected-capacity cost C",
+            "unit": "s / tok/s / GiB.s per request", "config": {
+                "workload": "12 synthetic documents, 16,078-67,744 tokens, arrivals every 0.5 s, <= 128 output tokens",
+                "fast_tier": "100 GiB, protected budget 50 GiB, 11 GiB/s staging, FCFS <= 4 active",
+                "retrieval_gbs": rates}, "results": out,
+            "model_seconds": round(_time.perf_counter() - t0, 2)}
+    print(json.dumps(line), flush=True)
+    return 0
+
+
 def main(argv=None):
     args = parse_args(argv)
+    if args.tempokv:
+        return run_tempokv(args)
     if args.impl == "reference":
         return run_reference(args)
     if args.overlap:
