@@ -4,16 +4,16 @@
 // A call is planned on the host: every (request, chunk) pair becomes one
 // Entry, every block of a chunk one physical block id, and the 2L plane
 // pointers one table.  The three arrays go to the device in one upload (a
-// pinned slot copied on the caller's stream), then one kernel per source class
-// moves the bytes:
-//   device-resident chunks  -> LDG or TMA kernel, HBM to HBM;
+// pinned slot copied on the caller's stream), then one launch per source class
+// (per layer group, for layer-wise calls) moves the bytes:
+//   device-resident chunks  -> LDG or TMA kernel, HBM to HBM (on a library
+//                              stream joined back when host chunks run too);
 //   host-resident chunks    -> HOSTLINK: a double-buffered vector kernel loads/stores
 //                              host memory over the host link directly, or
 //                              HBMCOPY: the copy engine moves whole chunks
 //                              through a ring of HBM staging slots and the
 //                              device kernel scatters/gathers from there.
 #include <algorithm>
-#include <chrono>
 #include <cstdarg>
 #include <cstdio>
 #include <cstring>

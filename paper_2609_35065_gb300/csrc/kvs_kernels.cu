@@ -399,16 +399,25 @@ Decoder make_decoder(const Job& job) {
     return dc;
 }
 
-int g_sms = 0;
+// Per-device facts, looked up once per device (a process may drive several GPUs).
+constexpr int kMaxDevices = 64;
+int g_sms[kMaxDevices];
+size_t g_tma_smem[kMaxDevices];          // dynamic shared memory the TMA kernel may use
+
+int current_device() {
+    int dev = 0;
+    cudaGetDevice(&dev);
+    return (dev >= 0 && dev < kMaxDevices) ? dev : 0;
+}
 
 int num_sms() {
-    if (g_sms == 0) {
-        int dev = 0;
-        cudaGetDevice(&dev);
-        cudaDeviceGetAttribute(&g_sms, cudaDevAttrMultiProcessorCount, dev);
-        if (g_sms <= 0) g_sms = 1;
+    const int dev = current_device();
+    if (g_sms[dev] == 0) {
+        int n = 0;
+        cudaDeviceGetAttribute(&n, cudaDevAttrMultiProcessorCount, dev);
+        g_sms[dev] = n > 0 ? n : 1;
     }
-    return g_sms;
+    return g_sms[dev];
 }
 
 int clamp_grid(int grid, int per_sm, uint64_t pieces) {
@@ -485,12 +494,12 @@ cudaError_t launch_ldg(const Job& job, int vec_bytes, int grid, cudaStream_t s) 
 cudaError_t launch_tma(const Job& job, int grid, cudaStream_t s) {
     if (job.num_pieces == 0) return cudaSuccess;
     const size_t smem = (size_t)kTmaStages * job.piece_bytes;
-    static size_t configured = 0;
-    if (configured < smem) {
+    const int dev = current_device();
+    if (g_tma_smem[dev] < smem) {             // the attribute is set per device
         cudaError_t e = cudaFuncSetAttribute(kvs_tma_kernel<kTmaStages>,
                                              cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
         if (e != cudaSuccess) return e;
-        configured = smem;
+        g_tma_smem[dev] = smem;
     }
     grid = clamp_grid(grid, tma_ctas_per_sm(), job.num_pieces);
     kvs_tma_kernel<kTmaStages><<<grid, 32, smem, s>>>(make_decoder(job), (uint32_t)job.num_pieces);
