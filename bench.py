@@ -653,7 +653,7 @@ def run_layerwise(args):
     def ev():
         return torch.cuda.Event(enable_timing=True)
 
-    def run(mode, lps=1):
+    def run(mode, lps=1, ctas=0):
         torch.cuda.synchronize()
         t0, t1 = ev(), ev()
         t0.record(main)
@@ -676,7 +676,8 @@ def run_layerwise(args):
         else:
             groups = -(-L // lps)
             evs = [ev() for _ in range(groups)]
-            kvs.kvs_retrieve_layers(g, buf.plane_ptrs, w.num_blocks, buf.requests, lps, evs, side, 0)
+            fl = (kvs.KVS_F_LAYER_LAUNCHES if mode == "launches" else 0) | kvs.KVS_F_MAX_CTAS(ctas)
+            kvs.kvs_retrieve_layers(g, buf.plane_ptrs, w.num_blocks, buf.requests, lps, evs, side, fl)
             for l in range(L):
                 if l % lps == 0:
                     main.wait_event(evs[l // lps])
@@ -685,15 +686,19 @@ def run_layerwise(args):
         torch.cuda.synchronize()
         return t0.elapsed_time(t1)
 
-    def best(mode, lps=1, reps=3):
-        run(mode, lps)
-        return min(run(mode, lps) for _ in range(reps))
+    def best(mode, lps=1, reps=3, ctas=0):
+        run(mode, lps, ctas)
+        return min(run(mode, lps, ctas) for _ in range(reps))
 
     res = {"retrieve_only_ms": best("retrieve"), "compute_only_ms": best("compute"),
            "serial_ms": best("serial")}
     for lps in (1, 4, 8):
-        res[f"layerwise_lps{lps}_ms"] = best("layer", lps)
-    pl = min(v for k, v in res.items() if k.startswith("layerwise"))
+        res[f"layerwise_lps{lps}_ms"] = best("layer", lps)                 # one signalling launch
+        res[f"layerwise_launches_lps{lps}_ms"] = best("launches", lps)     # one launch per group
+    for ctas in (4, 16):                                           # narrower copies
+        res[f"layerwise_lps1_ctas{ctas}_ms"] = best("layer", 1, ctas=ctas)
+    pl = min(v for k, v in res.items() if k.startswith("layerwise_lps") and "ctas" not in k)
+    pl_launches = min(v for k, v in res.items() if k.startswith("layerwise_launches") and "ctas" not in k)
     line = {"metric": METRIC + " (layer-wise retrieval pipelined with prefill compute)",
             "unit": "ms", "higher_is_better": False,
             "config": {"workload": describe(w), "compute": f"per layer one bf16 GEMM {M}x{K}x{N} "
@@ -703,6 +708,7 @@ def run_layerwise(args):
             "retrieval_gbs_alone": round(buf.payload_bytes / (res["retrieve_only_ms"] / 1e3) / 1e9, 2),
             "exposed_retrieval_ms_serial": round(res["serial_ms"] - res["compute_only_ms"], 3),
             "exposed_retrieval_ms_layerwise": round(pl - res["compute_only_ms"], 3),
+            "exposed_retrieval_ms_layer_launches": round(pl_launches - res["compute_only_ms"], 3),
             "speedup_vs_serial": round(res["serial_ms"] / pl, 4)}
     print(json.dumps(line), flush=True)
     return 0

@@ -81,6 +81,8 @@ extern "C" {
 #define KVS_F_FORCE_TMA      (1u << 4) /* kernel flavour: bulk async copies (TMA) staged
                                           through shared memory; 16-byte aligned data only  */
 #define KVS_F_NO_DEDUP       (1u << 5) /* write shared physical blocks once per request      */
+#define KVS_F_LAYER_LAUNCHES (1u << 6) /* layer-wise calls: one launch per layer group
+                                          instead of one signalling launch                 */
 #define KVS_F_MAX_CTAS(n)    ((((uint32_t)(n)) & 0xFFFFu) << 16) /* cap on CTAs, 0 = auto */
 #define KVS_F_GET_MAX_CTAS(f) (((f) >> 16) & 0xFFFFu)
 
@@ -169,6 +171,14 @@ int kvs_store(const kvs_geometry* geom, const kvs_paged_cache* cache,
  * layer_events may be NULL, and so may any of its entries; the events are the
  * caller's (cudaEvent_t cast to void*).  Host-resident chunks always take the
  * host-link kernel here (KVS_F_FORCE_HBMCOPY returns KVS_ERR_UNSUPPORTED).
+ * When every chunk is host-resident and events are given, the copy is ONE
+ * launch that stays resident and publishes each group's completion in device
+ * flags; a library stream waits on those flags (driver stream memory
+ * operations) and records layer_events[k] as group k lands, so group k's
+ * consumers never wait for a later launch to find free SMs.  Otherwise, or
+ * with KVS_F_LAYER_LAUNCHES, each group is its own launch followed by its
+ * event on cuda_stream.  Either way cuda_stream reaches the end of the whole
+ * copy after it.
  */
 int kvs_retrieve_layers(const kvs_geometry* geom, const kvs_paged_cache* cache,
                         const kvs_request* requests, int32_t num_requests,

@@ -21,6 +21,8 @@
 #include <string>
 #include <vector>
 
+#include <cuda.h>
+
 #include "kvs.h"
 #include "kvs_internal.h"
 
@@ -47,6 +49,7 @@ int fail(int code, const char* fmt, ...) {
     } while (0)
 
 constexpr int kUploadSlots = 4;
+constexpr int kSignalSlots = 4;
 constexpr int kRingSlots = 4;
 constexpr uint64_t kRingMinSlotBytes = 64ull << 20;
 
@@ -57,6 +60,17 @@ struct UploadSlot {
     cudaEvent_t done = nullptr;   // recorded after the last kernel that reads `dev`
     bool        used = false;
 };
+
+// Flags of one layer-wise signalling call: [ctas_done][counters x cap][flags x cap].
+struct SignalSlot {
+    uint32_t*   mem = nullptr;
+    uint32_t    cap = 0;          // groups
+    uint32_t    gen = 0;
+    cudaEvent_t done = nullptr;   // recorded after the kernel that uses `mem`
+    bool        used = false;
+};
+
+using WaitValueFn = CUresult (*)(CUstream, CUdeviceptr, cuuint32_t, unsigned int);
 
 struct DevState {
     bool         ready = false;
@@ -76,6 +90,12 @@ struct DevState {
     // device-resident chunks run on this stream, beside the host-resident ones
     cudaStream_t aux_stream = nullptr;
     cudaEvent_t  ev_aux_fork = nullptr, ev_aux_join = nullptr;
+    // layer-wise signalling: flags written by the copy kernel, waited on by this
+    // stream (stream memory operations), which then records the caller's events
+    cudaStream_t signal_stream = nullptr;
+    SignalSlot   sig[kSignalSlots];
+    int          next_sig = 0;
+    WaitValueFn  wait_value = nullptr;
     // per-block ownership for de-duplication: stamp[b] == gen -> owner[b] valid
     std::vector<uint32_t> stamp;
     std::vector<int64_t>  owner;
@@ -113,6 +133,16 @@ int get_state(DevState** out) {
         KVS_CUDA(cudaEventCreateWithFlags(&st.ev_fork, cudaEventDisableTiming));
         KVS_CUDA(cudaEventCreateWithFlags(&st.ev_join, cudaEventDisableTiming));
         KVS_CUDA(cudaStreamCreateWithFlags(&st.aux_stream, cudaStreamNonBlocking));
+        KVS_CUDA(cudaStreamCreateWithFlags(&st.signal_stream, cudaStreamNonBlocking));
+        for (auto& sg : st.sig) KVS_CUDA(cudaEventCreateWithFlags(&sg.done, cudaEventDisableTiming));
+        {
+            void* fn = nullptr;
+            cudaDriverEntryPointQueryResult q{};
+            if (cudaGetDriverEntryPointByVersion("cuStreamWaitValue32", &fn, 12000, cudaEnableDefault, &q)
+                    == cudaSuccess && q == cudaDriverEntryPointSuccess)
+                st.wait_value = (WaitValueFn)fn;
+            cudaGetLastError();
+        }
         KVS_CUDA(cudaEventCreateWithFlags(&st.ev_aux_fork, cudaEventDisableTiming));
         KVS_CUDA(cudaEventCreateWithFlags(&st.ev_aux_join, cudaEventDisableTiming));
         // Until kvs_query_bw measures them, host-link kernels take a third of the
@@ -571,6 +601,59 @@ int copy_call(const kvs_geometry* g, const kvs_paged_cache* cache, const kvs_req
     Uploaded u;
     rc = upload(st, pl, s, u);
     if (rc) return rc;
+    // Layer-wise, host chunks only: one persistent launch that publishes each
+    // group's completion; the signal stream waits on the flags and records the
+    // caller's events.  The kernel is enqueued before any wait, never waits on
+    // anything itself, and writes every flag before it ends.
+    if (layers_per_step > 0 && layer_events && !pl.num_device && vec == 16 && st.wait_value &&
+        !(flags & KVS_F_LAYER_LAUNCHES)) {
+        SignalSlot& sg = st.sig[st.next_sig];
+        st.next_sig = (st.next_sig + 1) % kSignalSlots;
+        if (sg.used) KVS_CUDA(cudaEventSynchronize(sg.done));
+        if (sg.cap < (uint32_t)groups) {
+            if (sg.mem) KVS_CUDA(cudaFree(sg.mem));
+            sg.mem = nullptr;
+            if (cudaMalloc(&sg.mem, (1 + 2 * (size_t)groups) * sizeof(uint32_t)) != cudaSuccess) {
+                cudaGetLastError();
+                sg.cap = 0;
+                return fail(KVS_ERR_NOMEM, "cannot allocate layer flags");
+            }
+            KVS_CUDA(cudaMemset(sg.mem, 0, (1 + 2 * (size_t)groups) * sizeof(uint32_t)));
+            sg.cap = (uint32_t)groups;
+            sg.gen = 0;
+        }
+        if (++sg.gen == 0) ++sg.gen;
+        Signal sig{sg.mem + 1, sg.mem + 1 + sg.cap, sg.mem, sg.gen, (uint32_t)groups, (uint32_t)(2 * lps)};
+        KVS_CUDA(cudaMemsetAsync(sg.mem, 0, (1 + (size_t)groups) * sizeof(uint32_t), s));
+        Job j = make_job(st, g, cache, pl, u, 0, pl.num_host, mode);
+        if (j.num_pieces) {
+            cudaError_t e = launch_link_signal(j, sig, host_grid, s);
+            if (e != cudaSuccess) return fail(KVS_ERR_CUDA, "kernel launch failed: %s", cudaGetErrorString(e));
+            ++g_launches;
+        }
+        KVS_CUDA(cudaEventRecord(sg.done, s));
+        sg.used = true;
+        bool waits_ok = j.num_pieces > 0;
+        for (int k = 0; k < groups; ++k) {
+            if (!layer_events[k]) continue;
+            if (waits_ok && st.wait_value((CUstream)st.signal_stream, (CUdeviceptr)(sig.flags + k), sig.gen,
+                                          CU_STREAM_WAIT_VALUE_GEQ) != CUDA_SUCCESS) {
+                st.wait_value = nullptr;            // not available here: events fire at kernel end
+                waits_ok = false;
+            }
+            KVS_CUDA(cudaEventRecord((cudaEvent_t)layer_events[k], waits_ok ? st.signal_stream : s));
+        }
+        if (!pl.blocks_cmp.empty()) {
+            Job jc = make_job(st, g, cache, pl, u, 0, (uint32_t)pl.entries.size(), MODE_COMPARE);
+            jc.blocks = u.blocks_cmp;
+            rc = launch_kernel(jc, KVS_KERNEL_LDG, vec, grid, s);
+            if (rc) return rc;
+        }
+        KVS_CUDA(cudaEventRecord(u.slot->done, s));
+        u.slot->used = true;
+        if (flags & KVS_F_VALIDATE) return read_error_word(st, s);
+        return KVS_OK;
+    }
     // With both classes present, the HBM-bound device part runs on the aux
     // stream while the link-bound host part runs on the caller's stream.
     const bool fork = pl.num_device && pl.num_host;
@@ -863,6 +946,11 @@ int kvs_shutdown(void) {
         cudaEventDestroy(st.ev_aux_fork);
         cudaEventDestroy(st.ev_aux_join);
         if (st.aux_stream) cudaStreamDestroy(st.aux_stream);
+        for (auto& sg : st.sig) {
+            if (sg.mem) cudaFree(sg.mem);
+            if (sg.done) cudaEventDestroy(sg.done);
+        }
+        if (st.signal_stream) cudaStreamDestroy(st.signal_stream);
         if (st.ring) cudaFree(st.ring);
         if (st.copy_stream) cudaStreamDestroy(st.copy_stream);
         if (st.err) cudaFree(st.err);

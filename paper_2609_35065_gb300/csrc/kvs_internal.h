@@ -57,6 +57,21 @@ cudaError_t launch_tma(const Job& job, int grid, cudaStream_t s);
 cudaError_t launch_link(const Job& job, int grid, cudaStream_t s);
 // Contiguous copy of `bytes` (multiple of 16, 16-byte aligned) for bandwidth probes.
 cudaError_t launch_flat_copy(void* dst, const void* src, uint64_t bytes, int grid, cudaStream_t s);
+// Layer-wise copy of host chunks in one launch: pieces go in plane-major
+// order, and the CTA that completes the last piece of layer group g writes
+// flags[g] = gen (after making the group's stores visible); the last CTA to
+// finish writes every flag, so all are written whatever the counts.  Consumers
+// wait on the flags with stream memory operations, not with kernels.
+struct Signal {
+    uint32_t* counters;        // per group: pieces done (zeroed before the launch)
+    uint32_t* flags;           // per group: generation of the last completed copy
+    uint32_t* ctas_done;       // CTAs finished (zeroed before the launch)
+    uint32_t  gen;
+    uint32_t  groups;
+    uint32_t  planes_per_group;
+};
+cudaError_t launch_link_signal(const Job& job, const Signal& sig, int grid, cudaStream_t s);
+
 // One CTA waits (bounded by limit_ns) on an mbarrier phase that nothing
 // completes, then records KVS_ERR_TIMEOUT: exercises the bounded-wait path.
 cudaError_t launch_stall(int32_t* err, uint64_t limit_ns, cudaStream_t s);

@@ -242,6 +242,88 @@ __global__ void __launch_bounds__(kLdgThreads) kvs_link_kernel(const Decoder dc,
     }
 }
 
+// Plane-major decode for the signalling kernel: q -> (plane, entry, block, piece).
+__device__ __forceinline__ bool decode_piece_plane_major(const Decoder& dc, const FastDiv& entries, uint32_t q,
+                                                         uint32_t& p_rel, Piece& pc) {
+    const Job& j = dc.job;
+    const uint32_t g = fdiv(q, dc.ppr);
+    const uint32_t k = q - g * dc.ppr.d;
+    const uint32_t g2 = fdiv(g, dc.bpc);
+    const uint32_t i = g - g2 * dc.bpc.d;
+    p_rel = fdiv(g2, entries);
+    const uint32_t e = g2 - p_rel * entries.d;
+    const uint32_t p = j.plane_begin + p_rel;
+    const int32_t blk = __ldg(j.blocks + (size_t)(j.entry_base + e) * j.blocks_per_chunk + i);
+    const Entry en = j.entries[e];
+    const int64_t first = (int64_t)i * j.block_size;
+    const int64_t ntok = min((int64_t)j.block_size, (int64_t)en.n_tok - first);
+    if (ntok <= 0 || blk < 0) return false;
+    if (blk >= j.num_blocks) {
+        atomicCAS(j.err, 0, KVS_ERR_BOUNDS);
+        return false;
+    }
+    const uint64_t run_bytes = (uint64_t)ntok * j.row_bytes;
+    const uint64_t off = (uint64_t)k * j.piece_bytes;
+    if (off >= run_bytes) return false;
+    pc.len = (uint32_t)min((uint64_t)j.piece_bytes, run_bytes - off);
+    pc.chunk_addr = en.chunk + ((uint64_t)p * (uint64_t)en.n_tok + (uint64_t)first) * j.row_bytes + off;
+    pc.plane_addr = j.planes[p] + (uint64_t)blk * j.block_size * j.row_bytes + off;
+    return true;
+}
+
+// Counts piece q as done; the CTA completing its group publishes the flag.
+__device__ __forceinline__ void piece_done(const Signal& sg, uint32_t p_rel, uint32_t group_pieces_full,
+                                           uint32_t last_group_pieces) {
+    __threadfence();                               // this thread's stores of the piece
+    __syncthreads();
+    if (threadIdx.x == 0) {
+        const uint32_t grp = p_rel / sg.planes_per_group;
+        const uint32_t total = (grp + 1 == sg.groups) ? last_group_pieces : group_pieces_full;
+        if (atomicAdd(&sg.counters[grp], 1u) + 1u == total) {
+            __threadfence();
+            atomicExch(&sg.flags[grp], sg.gen);
+        }
+    }
+}
+
+template <int MODE>
+__global__ void __launch_bounds__(kLdgThreads) kvs_link_signal_kernel(const Decoder dc, const FastDiv entries,
+                                                                      const Signal sg, uint32_t num_pieces) {
+    constexpr bool to_plane = (MODE == MODE_RETRIEVE);
+    const Job& j = dc.job;
+    const uint32_t per_plane = j.num_entries * j.blocks_per_chunk * j.pieces_per_run;
+    const uint32_t group_full = sg.planes_per_group * per_plane;
+    const uint32_t last_group = (j.num_planes - (sg.groups - 1) * sg.planes_per_group) * per_plane;
+    uint4 ra[kLdgUnroll], rb[kLdgUnroll];
+    Piece pa, pb;
+    uint32_t qa = blockIdx.x, qb, pra = 0, prb = 0;
+    bool ha = qa < num_pieces, va = false, vb = false;
+    if (ha && (va = decode_piece_plane_major(dc, entries, qa, pra, pa)))
+        load_piece16(to_plane ? pa.chunk_addr : pa.plane_addr, pa.len, ra);
+    while (ha) {
+        qb = qa + gridDim.x;
+        const bool hb = qb < num_pieces;
+        vb = hb && decode_piece_plane_major(dc, entries, qb, prb, pb);
+        if (vb) load_piece16(to_plane ? pb.chunk_addr : pb.plane_addr, pb.len, rb);
+        if (va) store_piece16(to_plane ? pa.plane_addr : pa.chunk_addr, pa.len, ra);
+        piece_done(sg, fdiv(fdiv(fdiv(qa, dc.ppr), dc.bpc), entries), group_full, last_group);
+        if (!hb) break;
+        qa = qb + gridDim.x;
+        ha = qa < num_pieces;
+        va = ha && decode_piece_plane_major(dc, entries, qa, pra, pa);
+        if (va) load_piece16(to_plane ? pa.chunk_addr : pa.plane_addr, pa.len, ra);
+        if (vb) store_piece16(to_plane ? pb.plane_addr : pb.chunk_addr, pb.len, rb);
+        piece_done(sg, fdiv(fdiv(fdiv(qb, dc.ppr), dc.bpc), entries), group_full, last_group);
+    }
+    // The last CTA to finish writes every flag (all groups are complete by then).
+    __syncthreads();
+    if (threadIdx.x == 0) {
+        __threadfence();
+        if (atomicAdd(sg.ctas_done, 1u) + 1u == gridDim.x)
+            for (uint32_t g = 0; g < sg.groups; ++g) atomicExch(&sg.flags[g], sg.gen);
+    }
+}
+
 __global__ void __launch_bounds__(kLdgThreads) kvs_flat_copy_kernel(uint64_t dst, uint64_t src, uint64_t bytes) {
     const uint64_t pieces = (bytes + kPieceBytes - 1) / kPieceBytes;
     for (uint64_t q = blockIdx.x; q < pieces; q += gridDim.x) {
@@ -508,6 +590,18 @@ cudaError_t launch_tma(const Job& job, int grid, cudaStream_t s) {
 
 cudaError_t launch_stall(int32_t* err, uint64_t limit_ns, cudaStream_t s) {
     kvs_stall_kernel<<<1, 32, 0, s>>>(err, limit_ns);
+    return cudaGetLastError();
+}
+
+cudaError_t launch_link_signal(const Job& job, const Signal& sig, int grid, cudaStream_t s) {
+    grid = clamp_grid(grid, link_ctas_per_sm(), std::max<uint64_t>(job.num_pieces, 1));
+    const Decoder dc = make_decoder(job);
+    const FastDiv entries = make_fastdiv(job.num_entries);
+    const uint32_t n = (uint32_t)job.num_pieces;
+    if (job.mode == MODE_RETRIEVE)
+        kvs_link_signal_kernel<MODE_RETRIEVE><<<grid, kLdgThreads, 0, s>>>(dc, entries, sig, n);
+    else
+        kvs_link_signal_kernel<MODE_STORE><<<grid, kLdgThreads, 0, s>>>(dc, entries, sig, n);
     return cudaGetLastError();
 }
 

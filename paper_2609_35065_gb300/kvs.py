@@ -42,6 +42,7 @@ KVS_F_FORCE_HBMCOPY = 1 << 2
 KVS_F_FORCE_LDG = 1 << 3
 KVS_F_FORCE_TMA = 1 << 4
 KVS_F_NO_DEDUP = 1 << 5
+KVS_F_LAYER_LAUNCHES = 1 << 6
 
 
 def KVS_F_MAX_CTAS(n: int) -> int:

@@ -29,9 +29,10 @@ def _workload(residency="host", L=6):
                         dist="normal", residency=residency)
 
 
+@pytest.mark.parametrize("flags", [0, kvs.KVS_F_LAYER_LAUNCHES], ids=["default", "launch_per_group"])
 @pytest.mark.parametrize("lps", [1, 2, 4, 6])
 @pytest.mark.parametrize("residency", ["host", "device", "mixed"])
-def test_layer_groups_are_ready_when_their_event_fires(lps, residency):
+def test_layer_groups_are_ready_when_their_event_fires(lps, residency, flags):
     res = ["host", "device", "host"] if residency == "mixed" else residency
     w = _workload(res)
     g = w.geom
@@ -39,7 +40,7 @@ def test_layer_groups_are_ready_when_their_event_fires(lps, residency):
     groups = -(-g.layers // lps)
     events = [torch.cuda.Event() for _ in range(groups)]
     copier, consumer = torch.cuda.Stream(), torch.cuda.Stream()
-    kvs.kvs_retrieve_layers(g, buf.plane_ptrs, w.num_blocks, buf.requests, lps, events, copier, 0)
+    kvs.kvs_retrieve_layers(g, buf.plane_ptrs, w.num_blocks, buf.requests, lps, events, copier, flags)
     snaps = []
     for k, ev in enumerate(events):
         consumer.wait_event(ev)
@@ -74,6 +75,7 @@ def test_layerwise_equals_whole_call_with_validation_and_shared_blocks():
 
 @pytest.mark.parametrize("lps", [1, 5])
 def test_store_layers_matches_oracle(lps):
+    """Host destinations with events: the signalling launch in the store direction."""
     w = synth.custom(5, 4, 64, 16, 256, 128, [1024, 700], [0, 0], seed=6, store_tokens=[768, 700])
     buf = buffers.allocate(w, store=True, plane_init="random")
     events = [torch.cuda.Event() for _ in range(-(-w.geom.layers // lps))]
