@@ -69,6 +69,8 @@ def workload(name: str):
         return synth.sweep(int(name[5:]) / 100.0)
     if name == "qwen14b":
         return synth.qwen14b()
+    if name == "qwen14b_small":          # profiling case: 2.25 GiB retrieved, 768 MiB stored, 3.2 GB planes
+        return synth.qwen14b(requests=1, num_blocks=1024)
     if name.startswith("llama70b"):
         frac = int(name.split("_")[1]) / 100.0 if "_" in name else 1.0
         return synth.llama70b(buffer_frac=frac)

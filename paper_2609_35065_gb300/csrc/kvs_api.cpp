@@ -377,6 +377,16 @@ struct Uploaded {
 
 size_t align_up(size_t x, size_t a) { return (x + a - 1) / a * a; }
 
+// Marks an upload slot in use on every exit path once its copy is enqueued:
+// the slot's event is recorded after everything the call enqueued on `s`.
+struct SlotGuard {
+    UploadSlot* slot = nullptr;
+    cudaStream_t s = nullptr;
+    ~SlotGuard() {
+        if (slot && cudaEventRecord(slot->done, s) == cudaSuccess) slot->used = true;
+    }
+};
+
 int upload(DevState& st, const Plan& pl, cudaStream_t s, Uploaded& u) {
     const size_t b_pl = align_up(pl.planes.size() * 8, 256);
     const size_t b_en = align_up(pl.entries.size() * sizeof(Entry), 256);
@@ -502,6 +512,7 @@ int run_hbmcopy(DevState& st, const kvs_geometry* g, const kvs_paged_cache* cach
     Uploaded ru;
     rc = upload(st, ring_plan, s, ru);
     if (rc) return rc;
+    SlotGuard ring_guard{ru.slot, s};
     const int vec = vec_bytes_for(ring_plan.addr_or);
     if (flavour == KVS_KERNEL_TMA && vec != 16) flavour = KVS_KERNEL_LDG;
 
@@ -535,8 +546,6 @@ int run_hbmcopy(DevState& st, const kvs_geometry* g, const kvs_paged_cache* cach
     }
     KVS_CUDA(cudaEventRecord(st.ev_join, st.copy_stream));
     KVS_CUDA(cudaStreamWaitEvent(s, st.ev_join, 0));
-    KVS_CUDA(cudaEventRecord(ru.slot->done, s));
-    ru.slot->used = true;
     return KVS_OK;
 }
 
@@ -601,6 +610,7 @@ int copy_call(const kvs_geometry* g, const kvs_paged_cache* cache, const kvs_req
     Uploaded u;
     rc = upload(st, pl, s, u);
     if (rc) return rc;
+    SlotGuard guard{u.slot, s};
     // Layer-wise, host chunks only: one persistent launch that publishes each
     // group's completion; the signal stream waits on the flags and records the
     // caller's events.  The kernel is enqueued before any wait, never waits on
@@ -649,9 +659,12 @@ int copy_call(const kvs_geometry* g, const kvs_paged_cache* cache, const kvs_req
             rc = launch_kernel(jc, KVS_KERNEL_LDG, vec, grid, s);
             if (rc) return rc;
         }
-        KVS_CUDA(cudaEventRecord(u.slot->done, s));
-        u.slot->used = true;
-        if (flags & KVS_F_VALIDATE) return read_error_word(st, s);
+        if (flags & KVS_F_VALIDATE) {
+            KVS_CUDA(cudaEventRecord(u.slot->done, s));   // before the synchronising read
+            u.slot->used = true;
+            guard.slot = nullptr;
+            return read_error_word(st, s);
+        }
         return KVS_OK;
     }
     // With both classes present, the HBM-bound device part runs on the aux
@@ -693,9 +706,12 @@ int copy_call(const kvs_geometry* g, const kvs_paged_cache* cache, const kvs_req
         rc = launch_kernel(j, KVS_KERNEL_LDG, vec, grid, s);
         if (rc) return rc;
     }
-    KVS_CUDA(cudaEventRecord(u.slot->done, s));
-    u.slot->used = true;
-    if (flags & KVS_F_VALIDATE) return read_error_word(st, s);
+    if (flags & KVS_F_VALIDATE) {
+        KVS_CUDA(cudaEventRecord(u.slot->done, s));       // before the synchronising read
+        u.slot->used = true;
+        guard.slot = nullptr;
+        return read_error_word(st, s);
+    }
     return KVS_OK;
 }
 

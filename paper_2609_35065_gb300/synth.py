@@ -125,7 +125,7 @@ def sweep(ratio: float, requests: int = 32, prompt: int = 8192) -> Workload:
 
 
 def qwen14b(requests: int = 8, prompt: int = 16384, hit: float = 0.75,
-            shared_frac: float = 0.10) -> Workload:
+            shared_frac: float = 0.10, num_blocks: int = 8192) -> Workload:
     """14B-shaped KV (48 layers, 8 KV heads, head_dim 128, 192 KiB/token), 8 requests
     of 16,384 tokens at 75% prefix hit; the 4096-token computed suffix is stored back
     into 256-token chunks.  The first 10% of each request's matched blocks are one
@@ -135,7 +135,7 @@ def qwen14b(requests: int = 8, prompt: int = 16384, hit: float = 0.75,
     nb_each = -(-prompt // B)
     matched = int(prompt * hit) // g.chunk_tokens * g.chunk_tokens
     shared_blocks = int(matched // B * shared_frac)
-    perm = _perm(8192, 0)
+    perm = _perm(num_blocks, 0)
     tables, at = [], 0
     for r in range(requests):
         if r == 0:
@@ -150,7 +150,8 @@ def qwen14b(requests: int = 8, prompt: int = 16384, hit: float = 0.75,
         raise ValueError("not enough blocks")
     reqs = [Request(prompt, matched, t, "host", store_tokens=prompt - matched,
                     shared_prefix_tokens=shared_blocks * B) for t in tables]
-    return Workload("qwen14b", g, 8192, reqs, notes={"shared_blocks": shared_blocks})
+    name = "qwen14b" if (requests, num_blocks) == (8, 8192) else f"qwen14b_r{requests}_nb{num_blocks}"
+    return Workload(name, g, num_blocks, reqs, notes={"shared_blocks": shared_blocks})
 
 
 def llama70b(requests: int = 4, prompt: int = 32768, buffer_frac: float = 1.0) -> Workload:
