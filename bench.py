@@ -418,7 +418,8 @@ def run_ours(args):
         peaks = measured_peaks()
         hpk = peaks.get("hbm_gbs", HBM_FALLBACK_GBS)
         ach = 2 * payload / (dms / 1e3) / 1e9
-        kname = "kvs_tma_kernel" if choice["chosen_kernel_device"] == 2 else "kvs_ldg_kernel"
+        tma = args.kernel == "tma" or (args.kernel == "auto" and choice["chosen_kernel_device"] == 2)
+        kname = "kvs_tma_kernel" if tma else "kvs_ldg_kernel"
         hbm = {"bound": "hbm", "achieved": round(ach, 1), "peak": hpk, "unit": "GB/s",
                "frac": round(ach / hpk, 4), "traffic": recorded_traffic(kname, "llama8b_device"),
                "kernel": kname, "payload_gbs": round(payload / (dms / 1e3) / 1e9, 1),

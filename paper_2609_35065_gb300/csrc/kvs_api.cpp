@@ -58,6 +58,7 @@ struct UploadSlot {
     void*       dev = nullptr;
     size_t      cap = 0;
     cudaEvent_t done = nullptr;   // recorded after the last kernel that reads `dev`
+    cudaEvent_t uploaded = nullptr;   // recorded after the host->device copy
     bool        used = false;
 };
 
@@ -80,6 +81,9 @@ struct DevState {
     int32_t*     err_host = nullptr;     // pinned read-back
     UploadSlot   up[kUploadSlots];
     int          next_up = 0;
+    // descriptor copies run here, so that a call's upload overlaps the kernels
+    // the caller's stream is still running
+    cudaStream_t upload_stream = nullptr;
     // HBM staging ring of the HBMCOPY variant
     uint8_t*     ring = nullptr;
     uint64_t     ring_slot_bytes = 0;
@@ -124,7 +128,11 @@ int get_state(DevState** out) {
         KVS_CUDA(cudaMalloc(&st.err, sizeof(int32_t)));
         KVS_CUDA(cudaMemset(st.err, 0, sizeof(int32_t)));
         KVS_CUDA(cudaHostAlloc(&st.err_host, sizeof(int32_t), cudaHostAllocDefault));
-        for (auto& s : st.up) KVS_CUDA(cudaEventCreateWithFlags(&s.done, cudaEventDisableTiming));
+        for (auto& s : st.up) {
+            KVS_CUDA(cudaEventCreateWithFlags(&s.done, cudaEventDisableTiming));
+            KVS_CUDA(cudaEventCreateWithFlags(&s.uploaded, cudaEventDisableTiming));
+        }
+        KVS_CUDA(cudaStreamCreateWithFlags(&st.upload_stream, cudaStreamNonBlocking));
         KVS_CUDA(cudaStreamCreateWithFlags(&st.copy_stream, cudaStreamNonBlocking));
         for (int k = 0; k < kRingSlots; ++k) {
             KVS_CUDA(cudaEventCreateWithFlags(&st.ring_filled[k], cudaEventDisableTiming));
@@ -413,7 +421,16 @@ int upload(DevState& st, const Plan& pl, cudaStream_t s, Uploaded& u) {
     memcpy(h + b_pl, pl.entries.data(), pl.entries.size() * sizeof(Entry));
     memcpy(h + b_pl + b_en, pl.blocks.data(), pl.blocks.size() * 4);
     if (b_bc) memcpy(h + b_pl + b_en + b_bl, pl.blocks_cmp.data(), pl.blocks_cmp.size() * 4);
-    KVS_CUDA(cudaMemcpyAsync(sl.dev, sl.host, need, cudaMemcpyHostToDevice, s));
+    // The slot's previous readers have finished (its `done` event, waited on
+    // above, follows them on the caller's stream), so the copy does not have to
+    // queue behind the caller's stream: only the kernels of this call wait for it.
+    KVS_CUDA(cudaMemcpyAsync(sl.dev, sl.host, need, cudaMemcpyHostToDevice, st.upload_stream));
+    cudaError_t e = cudaEventRecord(sl.uploaded, st.upload_stream);
+    if (e == cudaSuccess) e = cudaStreamWaitEvent(s, sl.uploaded, 0);
+    if (e != cudaSuccess) {
+        cudaStreamSynchronize(st.upload_stream);   // the slot is not tracked by `done`
+        return fail(KVS_ERR_CUDA, "descriptor upload: %s", cudaGetErrorString(e));
+    }
     uint8_t* d = (uint8_t*)sl.dev;
     u.planes = (const uint64_t*)d;
     u.entries = (const Entry*)(d + b_pl);
@@ -952,7 +969,9 @@ int kvs_shutdown(void) {
             if (sl.host) cudaFreeHost(sl.host);
             if (sl.dev) cudaFree(sl.dev);
             if (sl.done) cudaEventDestroy(sl.done);
+            if (sl.uploaded) cudaEventDestroy(sl.uploaded);
         }
+        if (st.upload_stream) cudaStreamDestroy(st.upload_stream);
         for (int k = 0; k < kRingSlots; ++k) {
             cudaEventDestroy(st.ring_filled[k]);
             cudaEventDestroy(st.ring_free[k]);
