@@ -419,7 +419,7 @@ def run_ours(args):
         hpk = peaks.get("hbm_gbs", HBM_FALLBACK_GBS)
         ach = 2 * payload / (dms / 1e3) / 1e9
         tma = args.kernel == "tma" or (args.kernel == "auto" and choice["chosen_kernel_device"] == 2)
-        kname = "kvs_tma_kernel" if tma else "kvs_ldg_kernel"
+        kname = "kvs_tma_kernel" if tma else ("kvs_ldg_kernel" if args.max_ctas else "kvs_ldg_piece_kernel")
         hbm = {"bound": "hbm", "achieved": round(ach, 1), "peak": hpk, "unit": "GB/s",
                "frac": round(ach / hpk, 4), "traffic": recorded_traffic(kname, "llama8b_device"),
                "kernel": kname, "payload_gbs": round(payload / (dms / 1e3) / 1e9, 1),
@@ -464,9 +464,14 @@ def run_ours(args):
         chunks_np = oracle_inputs_from_buffers(buf)
         cores = host_cores()
         secs = oracle_pass(w, chunks_np, cores)
+        sub = list(range(min(4, 2 * g.layers)))
+        secs1 = oracle_pass(w, chunks_np, 1, sub)
         cpu = {"value": round(payload / secs / 1e9, 3), "unit": "GB/s", "cores": cores, "kind": "oracle",
                "sample": f"one full pass of the workload ({payload} bytes, all {2 * g.layers} planes), "
-                         f"threads split by plane"}
+                         f"threads split by plane",
+               "single_thread": {"value": round(payload * len(sub) / (2 * g.layers) / secs1 / 1e9, 3),
+                                 "unit": "GB/s", "cores": 1,
+                                 "sample": f"planes 0-{len(sub) - 1} of {2 * g.layers} (same bytes per plane)"}}
 
     clocks = sampler.summary(wall0, wall1)
     mv = moved_bytes(w)
@@ -499,6 +504,9 @@ def run_ours(args):
                        "l2": f"inputs ({payload >> 20} MiB per step) larger than L2; no flush",
                        "parallelism": f"replicas x{world}"},
             "tokens_per_s": round(tokens_per_s, 1),
+            "per_step": {"best_ms": round(min(per_call_ms), 4), "median_ms": round(statistics.median(per_call_ms), 4),
+                         "best_gbs": round(payload / min(per_call_ms) / 1e6, 3),
+                         "median_gbs": round(payload / statistics.median(per_call_ms) / 1e6, 3)},
             "roofline": roofline,
             "roofline_hbm": hbm,
             "extras": extras or None,

@@ -685,21 +685,16 @@ int copy_call(const kvs_geometry* g, const kvs_paged_cache* cache, const kvs_req
         return KVS_OK;
     }
     // With both classes present, the HBM-bound device part runs on the aux
-    // stream while the link-bound host part runs on the caller's stream.
+    // stream while the link-bound host part runs on the caller's stream.  The
+    // host part is launched first: its few CTAs take their SM slots before the
+    // whole-GPU device grid fills every SM.
     const bool fork = pl.num_device && pl.num_host;
     for (int k = 0; k < groups; ++k) {
         const uint32_t p0 = (uint32_t)(2 * k * lps);
         const uint32_t np = (uint32_t)(2 * (std::min(L, (k + 1) * lps) - k * lps));
-        if (pl.num_device) {
-            cudaStream_t ds = s;
-            if (fork) {
-                KVS_CUDA(cudaEventRecord(st.ev_aux_fork, s));
-                KVS_CUDA(cudaStreamWaitEvent(st.aux_stream, st.ev_aux_fork, 0));
-                ds = st.aux_stream;
-            }
-            rc = launch_kernel(make_job(st, g, cache, pl, u, 0, pl.num_device, mode, p0, np), flavour, vec, grid, ds);
-            if (rc) return rc;
-            if (fork) KVS_CUDA(cudaEventRecord(st.ev_aux_join, st.aux_stream));
+        if (fork) {
+            KVS_CUDA(cudaEventRecord(st.ev_aux_fork, s));
+            KVS_CUDA(cudaStreamWaitEvent(st.aux_stream, st.ev_aux_fork, 0));
         }
         if (pl.num_host) {
             if (host_variant == KVS_VARIANT_HBMCOPY) {
@@ -712,6 +707,12 @@ int copy_call(const kvs_geometry* g, const kvs_paged_cache* cache, const kvs_req
                                    kKernelLink, vec, host_grid, s);
             }
             if (rc) return rc;
+        }
+        if (pl.num_device) {
+            const cudaStream_t ds = fork ? st.aux_stream : s;
+            rc = launch_kernel(make_job(st, g, cache, pl, u, 0, pl.num_device, mode, p0, np), flavour, vec, grid, ds);
+            if (rc) return rc;
+            if (fork) KVS_CUDA(cudaEventRecord(st.ev_aux_join, st.aux_stream));
         }
         if (fork) KVS_CUDA(cudaStreamWaitEvent(s, st.ev_aux_join, 0));
         if (layers_per_step > 0 && layer_events && layer_events[k])

@@ -189,6 +189,41 @@ __global__ void __launch_bounds__(kLdgThreads) kvs_ldg_kernel(const Decoder dc, 
     }
 }
 
+// Whole-GPU flavour for 16-byte aligned work: exactly one CTA per piece, 512
+// threads x 4 vectors.  The launch bound caps the kernel at 32 registers, so
+// four CTAs (2048 threads, 128 KiB of loads in flight) fit on an SM, twice the
+// residency of kvs_ldg_kernel<16>.
+constexpr int kPieceThreads = 512;
+constexpr int kPieceUnroll = kPieceBytes / 16 / kPieceThreads;
+
+template <int MODE>
+__global__ void __launch_bounds__(kPieceThreads, 4) kvs_ldg_piece_kernel(const Decoder dc) {
+    static_assert(kPieceUnroll * kPieceThreads * 16 == kPieceBytes, "one piece per CTA");
+    Piece pc;
+    if (!decode_piece(dc, blockIdx.x, pc)) return;       // uniform across the CTA
+    const uint4* s = reinterpret_cast<const uint4*>(MODE == MODE_RETRIEVE ? pc.chunk_addr : pc.plane_addr);
+    uint4* d = reinterpret_cast<uint4*>(MODE == MODE_RETRIEVE ? pc.plane_addr : pc.chunk_addr);
+    const uint32_t n = pc.len / 16;
+    uint4 r[kPieceUnroll];
+    if (n == kPieceThreads * kPieceUnroll) {
+#pragma unroll
+        for (int u = 0; u < kPieceUnroll; ++u) r[u] = ld_stream<16>(s + threadIdx.x + u * kPieceThreads);
+#pragma unroll
+        for (int u = 0; u < kPieceUnroll; ++u) st_stream<16>(d + threadIdx.x + u * kPieceThreads, r[u]);
+    } else {                                             // a short run: the tail of a partial chunk
+#pragma unroll
+        for (int u = 0; u < kPieceUnroll; ++u) {
+            const uint32_t k = threadIdx.x + u * kPieceThreads;
+            if (k < n) r[u] = ld_stream<16>(s + k);
+        }
+#pragma unroll
+        for (int u = 0; u < kPieceUnroll; ++u) {
+            const uint32_t k = threadIdx.x + u * kPieceThreads;
+            if (k < n) st_stream<16>(d + k, r[u]);
+        }
+    }
+}
+
 // Host-link flavour: each thread keeps two pieces' worth of 16-byte vectors in
 // registers, so the loads of the next piece are in flight while the current
 // one is stored.  A CTA then always has 32-64 KiB outstanding over the
@@ -515,9 +550,16 @@ int clamp_grid(int grid, int per_sm, uint64_t pieces) {
 // persistent grid-stride grids of any shape.
 template <int V>
 cudaError_t launch_ldg_v(const Job& job, int grid, cudaStream_t s) {
-    grid = grid > 0 ? clamp_grid(grid, ldg_ctas_per_sm(), job.num_pieces) : (int)job.num_pieces;
     const Decoder dc = make_decoder(job);
     const uint32_t n = (uint32_t)job.num_pieces;
+    if (V == 16 && grid <= 0 && job.mode != MODE_COMPARE) {
+        if (job.mode == MODE_RETRIEVE)
+            kvs_ldg_piece_kernel<MODE_RETRIEVE><<<n, kPieceThreads, 0, s>>>(dc);
+        else
+            kvs_ldg_piece_kernel<MODE_STORE><<<n, kPieceThreads, 0, s>>>(dc);
+        return cudaGetLastError();
+    }
+    grid = grid > 0 ? clamp_grid(grid, ldg_ctas_per_sm(), job.num_pieces) : (int)job.num_pieces;
     if (job.mode == MODE_RETRIEVE)
         kvs_ldg_kernel<V, MODE_RETRIEVE><<<grid, kLdgThreads, 0, s>>>(dc, n);
     else if (job.mode == MODE_STORE)
