@@ -82,7 +82,9 @@ extern "C" {
                                           through shared memory; 16-byte aligned data only  */
 #define KVS_F_NO_DEDUP       (1u << 5) /* write shared physical blocks once per request      */
 #define KVS_F_LAYER_LAUNCHES (1u << 6) /* layer-wise calls: one launch per layer group
-                                          instead of one signalling launch                 */
+                                          (the default; accepted for explicitness)         */
+#define KVS_F_LAYER_SIGNAL   (1u << 7) /* layer-wise calls: one resident launch that
+                                          signals each group (see kvs_retrieve_layers)     */
 #define KVS_F_MAX_CTAS(n)    ((((uint32_t)(n)) & 0xFFFFu) << 16) /* cap on CTAs, 0 = auto */
 #define KVS_F_GET_MAX_CTAS(f) (((f) >> 16) & 0xFFFFu)
 
@@ -171,14 +173,18 @@ int kvs_store(const kvs_geometry* geom, const kvs_paged_cache* cache,
  * layer_events may be NULL, and so may any of its entries; the events are the
  * caller's (cudaEvent_t cast to void*).  Host-resident chunks always take the
  * host-link kernel here (KVS_F_FORCE_HBMCOPY returns KVS_ERR_UNSUPPORTED).
- * When every chunk is host-resident and events are given, the copy is ONE
- * launch that stays resident and publishes each group's completion in device
- * flags; a library stream waits on those flags (driver stream memory
- * operations) and records layer_events[k] as group k lands, so group k's
- * consumers never wait for a later launch to find free SMs.  Otherwise, or
- * with KVS_F_LAYER_LAUNCHES, each group is its own launch followed by its
- * event on cuda_stream.  Either way cuda_stream reaches the end of the whole
- * copy after it.
+ * By default each group is its own launch followed by its event on
+ * cuda_stream: between groups the SMs go back to whatever else runs (the
+ * model's compute), so the copy keeps just ahead of its consumer without a
+ * tuned CTA cap.  With KVS_F_LAYER_SIGNAL, when every chunk is host-resident
+ * and 16-byte aligned and events are given, the copy is instead ONE launch
+ * that stays resident and publishes each group's completion in device flags;
+ * a library stream waits on those flags (driver stream memory operations) and
+ * records layer_events[k] as group k lands (otherwise the call falls back to
+ * per-group launches).  A resident launch holds its SMs for the whole copy,
+ * so it suits a small KVS_F_MAX_CTAS cap.  KVS_F_LAYER_LAUNCHES together with
+ * KVS_F_LAYER_SIGNAL is KVS_ERR_INVALID_ARG.  Either way cuda_stream reaches
+ * the end of the whole copy after it.
  */
 int kvs_retrieve_layers(const kvs_geometry* geom, const kvs_paged_cache* cache,
                         const kvs_request* requests, int32_t num_requests,
@@ -389,7 +395,7 @@ void* kvs_tier_slot(const kvs_tier* tier, int64_t slot);
 
 /* ABI version of this header: major * 10000 + minor * 100 + patch. */
 int kvs_version(void);
-#define KVS_VERSION 10300
+#define KVS_VERSION 10400
 
 #ifdef __cplusplus
 }

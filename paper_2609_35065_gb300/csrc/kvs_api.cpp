@@ -588,6 +588,8 @@ int copy_call(const kvs_geometry* g, const kvs_paged_cache* cache, const kvs_req
     const bool f_ldg = flags & KVS_F_FORCE_LDG, f_tma = flags & KVS_F_FORCE_TMA;
     if ((f_host && f_hbm) || (f_ldg && f_tma))
         return fail(KVS_ERR_INVALID_ARG, "conflicting FORCE flags");
+    if ((flags & KVS_F_LAYER_LAUNCHES) && (flags & KVS_F_LAYER_SIGNAL))
+        return fail(KVS_ERR_INVALID_ARG, "KVS_F_LAYER_LAUNCHES and KVS_F_LAYER_SIGNAL together");
     if (layers_per_step < 0) return fail(KVS_ERR_INVALID_ARG, "layers_per_step must be positive");
     if (layers_per_step > 0 && f_hbm)
         return fail(KVS_ERR_UNSUPPORTED, "layer-wise copies move host chunks over the host link only");
@@ -633,7 +635,7 @@ int copy_call(const kvs_geometry* g, const kvs_paged_cache* cache, const kvs_req
     // caller's events.  The kernel is enqueued before any wait, never waits on
     // anything itself, and writes every flag before it ends.
     if (layers_per_step > 0 && layer_events && !pl.num_device && vec == 16 && st.wait_value &&
-        !(flags & KVS_F_LAYER_LAUNCHES)) {
+        (flags & KVS_F_LAYER_SIGNAL)) {
         SignalSlot& sg = st.sig[st.next_sig];
         st.next_sig = (st.next_sig + 1) % kSignalSlots;
         if (sg.used) KVS_CUDA(cudaEventSynchronize(sg.done));

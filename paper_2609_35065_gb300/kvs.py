@@ -43,6 +43,7 @@ KVS_F_FORCE_LDG = 1 << 3
 KVS_F_FORCE_TMA = 1 << 4
 KVS_F_NO_DEDUP = 1 << 5
 KVS_F_LAYER_LAUNCHES = 1 << 6
+KVS_F_LAYER_SIGNAL = 1 << 7
 
 
 def KVS_F_MAX_CTAS(n: int) -> int:

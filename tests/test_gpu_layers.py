@@ -29,7 +29,8 @@ def _workload(residency="host", L=6):
                         dist="normal", residency=residency)
 
 
-@pytest.mark.parametrize("flags", [0, kvs.KVS_F_LAYER_LAUNCHES], ids=["default", "launch_per_group"])
+@pytest.mark.parametrize("flags", [0, kvs.KVS_F_LAYER_SIGNAL, kvs.KVS_F_LAYER_SIGNAL | kvs.KVS_F_MAX_CTAS(4)],
+                         ids=["launch_per_group", "signal", "signal_4ctas"])
 @pytest.mark.parametrize("lps", [1, 2, 4, 6])
 @pytest.mark.parametrize("residency", ["host", "device", "mixed"])
 def test_layer_groups_are_ready_when_their_event_fires(lps, residency, flags):
