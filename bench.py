@@ -395,7 +395,7 @@ def run_ours(args):
            "ms_per_step": round(e2e_s * 1e3, 3)}
 
     # device-resident (HBM staging) source, same workload: the HBM roofline
-    hbm = None
+    hbm = hbm_store = None
     if rank == 0 and w.name.startswith("llama8b"):
         dpool = torch.empty_like(buf.host_pool, device="cuda")
         dpool.copy_(buf.host_pool)
@@ -426,12 +426,35 @@ def run_ours(args):
         hpk = peaks.get("hbm_gbs", HBM_FALLBACK_GBS)
         ach = 2 * payload / (dms / 1e3) / 1e9
         tma = args.kernel == "tma" or (args.kernel == "auto" and choice["chosen_kernel_device"] == 2)
-        kname = "kvs_tma_kernel" if tma else ("kvs_ldg_kernel" if args.max_ctas else "kvs_ldg_piece_kernel")
+        if args.max_ctas:
+            kname = "kvs_tma_kernel" if tma else "kvs_ldg_kernel"
+        else:
+            kname = "kvs_tma_piece_kernel" if tma else "kvs_ldg_piece_kernel"
         hbm = {"bound": "hbm", "achieved": round(ach, 1), "peak": hpk, "unit": "GB/s",
                "frac": round(ach / hpk, 4), "traffic": recorded_traffic(kname, "llama8b_device"),
                "kernel": kname, "payload_gbs": round(payload / (dms / 1e3) / 1e9, 1),
                "peak_source": "MEASURED_PEAKS.json hbm_gbs (copy, read+write bytes)" if peaks else "fallback",
                "bytes_counted": "2 x payload (read + write)"}
+
+        # store-back (gather) of the same blocks into the HBM-resident chunks
+        def sstep(f=dflags):
+            kvs.kvs_store(g, buf.plane_ptrs, w.num_blocks, dreqs, stream, f)
+        sstep(dflags | kvs.KVS_F_VALIDATE)
+        for _ in range(3):
+            sstep()
+        torch.cuda.synchronize()
+        st_ev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)) for _ in range(nd)]
+        for a, b in st_ev:
+            a.record(stream)
+            sstep()
+            b.record(stream)
+        torch.cuda.synchronize()
+        sms = statistics.mean(a.elapsed_time(b) for a, b in st_ev)
+        sach = 2 * payload / (sms / 1e3) / 1e9
+        hbm_store = {"bound": "hbm", "achieved": round(sach, 1), "peak": hpk, "unit": "GB/s",
+                     "frac": round(sach / hpk, 4), "traffic": None, "kernel": kname,
+                     "payload_gbs": round(payload / (sms / 1e3) / 1e9, 1),
+                     "bytes_counted": "2 x payload (read + write)"}
         del dpool
 
     def timed_calls(fn, n):
@@ -516,6 +539,7 @@ def run_ours(args):
                          "median_gbs": round(payload / statistics.median(per_call_ms) / 1e6, 3)},
             "roofline": roofline,
             "roofline_hbm": hbm,
+            "roofline_hbm_store": hbm_store,
             "extras": extras or None,
             "cpu_baseline": cpu,
             "e2e": e2e,

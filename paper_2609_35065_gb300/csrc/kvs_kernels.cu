@@ -498,6 +498,33 @@ __global__ void __launch_bounds__(32, 1) kvs_tma_kernel(const Decoder dc, uint32
     bulk_wait_all();
 }
 
+// Whole-GPU TMA flavour: exactly one 32-thread CTA per piece; its elected
+// thread moves the piece through 32 KiB of shared memory with one bulk load
+// (completing on an mbarrier, bounded wait) and one bulk store, and leaves once
+// the store has read the stage.  Shared memory allows six such CTAs per SM,
+// 192 KiB of loads in flight, with almost no registers.
+template <int MODE>
+__global__ void __launch_bounds__(32) kvs_tma_piece_kernel(const Decoder dc) {
+    extern __shared__ __align__(128) uint8_t stage[];
+    __shared__ __align__(8) uint64_t bar;
+    if (threadIdx.x != 0) return;
+    Piece pc;
+    if (!decode_piece(dc, blockIdx.x, pc)) return;
+    const uint32_t b = smem_u32(&bar);
+    mbar_init(b, 1);
+    asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+    mbar_expect_tx(b, pc.len);
+    bulk_load(smem_u32(stage), MODE == MODE_RETRIEVE ? pc.chunk_addr : pc.plane_addr, pc.len, b);
+    if (!mbar_wait(b, 0, kWaitLimitNs)) {
+        atomicCAS(dc.job.err, 0, KVS_ERR_TIMEOUT);
+        mbar_wait(b, 0, kWaitLimitNs);             // let the load land before the stage goes away
+        return;
+    }
+    bulk_store(MODE == MODE_RETRIEVE ? pc.plane_addr : pc.chunk_addr, smem_u32(stage), pc.len);
+    bulk_commit();
+    bulk_wait_read<0>();
+}
+
 // Waits on a barrier phase that nothing completes; the bounded wait must give up.
 __global__ void kvs_stall_kernel(int32_t* err, uint64_t limit_ns) {
     __shared__ __align__(8) uint64_t bar;
@@ -520,6 +547,7 @@ Decoder make_decoder(const Job& job) {
 constexpr int kMaxDevices = 64;
 int g_sms[kMaxDevices];
 size_t g_tma_smem[kMaxDevices];          // dynamic shared memory the TMA kernel may use
+bool g_tma_piece_cfg[kMaxDevices];       // carveout preference of the per-piece TMA kernel set
 
 int current_device() {
     int dev = 0;
@@ -617,8 +645,27 @@ cudaError_t launch_ldg(const Job& job, int vec_bytes, int grid, cudaStream_t s) 
 
 cudaError_t launch_tma(const Job& job, int grid, cudaStream_t s) {
     if (job.num_pieces == 0) return cudaSuccess;
-    const size_t smem = (size_t)kTmaStages * job.piece_bytes;
     const int dev = current_device();
+    if (grid <= 0 && job.mode != MODE_COMPARE) {
+        // The carveout preference asks for the largest shared-memory split, so
+        // that six 33 KiB CTAs (stage + reserved) fit on an SM.
+        if (!g_tma_piece_cfg[dev]) {
+            for (auto fn : {kvs_tma_piece_kernel<MODE_RETRIEVE>, kvs_tma_piece_kernel<MODE_STORE>}) {
+                cudaError_t e = cudaFuncSetAttribute(fn, cudaFuncAttributePreferredSharedMemoryCarveout,
+                                                     (int)cudaSharedmemCarveoutMaxShared);
+                if (e != cudaSuccess) return e;
+            }
+            g_tma_piece_cfg[dev] = true;
+        }
+        const Decoder dc = make_decoder(job);
+        const uint32_t n = (uint32_t)job.num_pieces;
+        if (job.mode == MODE_RETRIEVE)
+            kvs_tma_piece_kernel<MODE_RETRIEVE><<<n, 32, job.piece_bytes, s>>>(dc);
+        else
+            kvs_tma_piece_kernel<MODE_STORE><<<n, 32, job.piece_bytes, s>>>(dc);
+        return cudaGetLastError();
+    }
+    const size_t smem = (size_t)kTmaStages * job.piece_bytes;
     if (g_tma_smem[dev] < smem) {             // the attribute is set per device
         cudaError_t e = cudaFuncSetAttribute(kvs_tma_kernel<kTmaStages>,
                                              cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
