@@ -452,7 +452,8 @@ def run_ours(args):
         sms = statistics.mean(a.elapsed_time(b) for a, b in st_ev)
         sach = 2 * payload / (sms / 1e3) / 1e9
         hbm_store = {"bound": "hbm", "achieved": round(sach, 1), "peak": hpk, "unit": "GB/s",
-                     "frac": round(sach / hpk, 4), "traffic": None, "kernel": kname,
+                     "frac": round(sach / hpk, 4), "traffic": recorded_traffic(kname, "llama8b_device_store"),
+                     "kernel": kname,
                      "payload_gbs": round(payload / (sms / 1e3) / 1e9, 1),
                      "bytes_counted": "2 x payload (read + write)"}
         del dpool
