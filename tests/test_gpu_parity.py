@@ -123,6 +123,28 @@ def test_random_small_geometries(seed):
     gc.check_store(buf)
 
 
+@pytest.mark.parametrize("kernel", ["ldg", "tma"])
+@pytest.mark.parametrize("geometry", [(2, 8, 256), (3, 4, 128)], ids=["64KiB_runs", "16KiB_runs"])
+def test_per_piece_kernels_full_and_partial_pieces(kernel, geometry):
+    """Uncapped HBM copies run one CTA per 32 KiB piece.  With H8 D256 a block's run is
+    64 KiB (two pieces); with H4 D128 it is 16 KiB (one short piece).  The 700-token
+    request ends in a 188-token chunk whose last block holds 12 tokens, so full pieces,
+    partial pieces and partial blocks all occur, in both directions."""
+    L, H, D = geometry
+    flags = kvs.KVS_F_FORCE_LDG if kernel == "ldg" else kvs.KVS_F_FORCE_TMA
+    w = synth.custom(L, H, D, 16, 256, 300, [1024, 700, 512], [1024, 700, 512], seed=5, dist="normal",
+                     residency="device")
+    buf = buffers.allocate(w)
+    _retrieve(buf, flags)
+    torch.cuda.synchronize()
+    gc.check_retrieve(buf)
+    ws = synth.custom(L, H, D, 16, 256, 300, [1024, 700], [0, 0], seed=6, store_tokens=[1024, 700])
+    sbuf = buffers.allocate(ws, store=True, store_residency="device", plane_init="random")
+    _store(sbuf, flags)
+    torch.cuda.synchronize()
+    gc.check_store(sbuf)
+
+
 def test_tma_rejects_unaligned_rows():
     w = synth.custom(1, 3, 5, 4, 8, 8, [16], [16])            # 30-byte rows
     w.requests[0].residency = "device"
