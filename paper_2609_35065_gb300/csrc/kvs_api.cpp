@@ -4,7 +4,8 @@
 // A call is planned on the host: every (request, chunk) pair becomes one
 // Entry, every block of a chunk one physical block id, and the 2L plane
 // pointers one table.  The three arrays go to the device in one upload (a
-// pinned slot copied on the caller's stream), then one launch per source class
+// pinned slot copied on a library stream that the caller's stream waits on),
+// then one launch per source class
 // (per layer group, for layer-wise calls) moves the bytes:
 //   device-resident chunks  -> LDG or TMA kernel, HBM to HBM (on a library
 //                              stream joined back when host chunks run too);

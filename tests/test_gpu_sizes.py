@@ -36,13 +36,17 @@ def test_llama8b_host_source(flags):
     gc.free(buf)
 
 
-@pytest.mark.parametrize("ratio", [25, 50, 75])
-def test_sweep_mixed_residency(ratio):
+@pytest.mark.parametrize("ratio,flags", [(25, 0), (50, 0), (75, 0), (50, kvs.KVS_F_FORCE_TMA),
+                                         (50, kvs.KVS_F_FORCE_LDG)],
+                         ids=["25", "50", "75", "50_tma", "50_ldg"])
+def test_sweep_mixed_residency(ratio, flags):
+    """Host class on the host-link kernel, HBM class (one CTA per piece, LDG or TMA)
+    beside it on a second stream."""
     w = synth.sweep(ratio / 100)
     res = {r.residency for r in w.requests}
     assert res == {"host", "device"}
     buf = buffers.allocate(w)
-    _run(buf)
+    _run(buf, flags=flags)
     torch.cuda.synchronize()
     gc.check_retrieve(buf)
     gc.free(buf)
