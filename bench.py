@@ -715,7 +715,9 @@ def run_layerwise(args):
     kvs.kvs_query_bw(side, 1 << 30)
     w = workload(args.config)
     g = w.geom
-    buf = buffers.allocate(w)
+    for r in w.requests:                  # the computed suffix is stored back into chunks
+        r.store_tokens = r.prompt_tokens - r.matched_tokens
+    buf = buffers.allocate(w, store=True)
     suffix = sum(r.prompt_tokens - r.matched_tokens for r in w.requests)
     # per-layer prefill work of the suffix: q/k/v + o + gated MLP widths of Llama-3-8B
     M, K, N = suffix, 4096, (4096 + 2 * 1024) + 4096 + 3 * 14336
@@ -747,6 +749,27 @@ def run_layerwise(args):
             done = ev()
             done.record(side)
             main.wait_event(done)
+        elif mode == "store_serial":
+            for _ in range(L):
+                torch.matmul(a, b, out=c)
+            computed = ev()
+            computed.record(main)
+            side.wait_event(computed)
+            kvs.kvs_store(g, buf.plane_ptrs, w.num_blocks, buf.store_requests, side, 0)
+            done = ev()
+            done.record(side)
+            main.wait_event(done)
+        elif mode == "store_layer":
+            ready = []
+            for _ in range(L):
+                torch.matmul(a, b, out=c)
+                ready.append(ev())
+                ready[-1].record(main)
+            kvs.kvs_store_layers(g, buf.plane_ptrs, w.num_blocks, buf.store_requests, lps, None, side,
+                                 kvs.KVS_F_MAX_CTAS(ctas), ready_events=ready[lps - 1::lps] if lps > 1 else ready)
+            done = ev()
+            done.record(side)
+            main.wait_event(done)
         else:
             groups = -(-L // lps)
             evs = [ev() for _ in range(groups)]
@@ -763,7 +786,10 @@ def run_layerwise(args):
                  ("layerwise_lps1", "layer", 1, 0), ("layerwise_lps4", "layer", 4, 0),
                  ("layerwise_lps8", "layer", 8, 0), ("layerwise_lps1_ctas4", "layer", 1, 4),
                  ("layerwise_signal_lps1", "signal", 1, 0), ("layerwise_signal_lps1_ctas4", "signal", 1, 4),
-                 ("layerwise_signal_lps1_ctas16", "signal", 1, 16)]
+                 ("layerwise_signal_lps1_ctas16", "signal", 1, 16),
+                 # store-back of the computed suffix: after the whole prefill, or layer by layer
+                 ("store_serial", "store_serial", 1, 0), ("store_layerwise_lps1", "store_layer", 1, 0),
+                 ("store_layerwise_lps1_ctas4", "store_layer", 1, 4)]
     reps = max(3, min(args.steps, 10))
     sampler = ClockSampler(0)
     time.sleep(0.2)
@@ -779,34 +805,62 @@ def run_layerwise(args):
         t1.record(main)
         torch.cuda.synchronize()
         retrieve_alone.append(t0.elapsed_time(t1))
+    def block(mode, lps, ctas):
+        one(mode, lps, ctas)                              # settle into this schedule
+        t0, t1 = ev(), ev()
+        t0.record(main)
+        w0 = time.time()
+        for _ in range(reps):
+            one(mode, lps, ctas)
+        t1.record(main)
+        torch.cuda.synchronize()
+        return t0.elapsed_time(t1) / reps, sampler.summary(w0 + 0.3, time.time())
+
+    # compute-only blocks bracket every schedule (C S1 C S2 C ...); a schedule's
+    # exposed copy time is taken against the mean of its two neighbours, which
+    # cancels the slow drift of the power-capped clock
+    exposed = {name: [] for name, *_ in schedules if name != "compute_only"}
     for _pass in range(2):
+        before, clk = block("compute", 1, 0)
+        times["compute_only"].append(before)
+        clocks["compute_only"].append(clk)
         for name, mode, lps, ctas in schedules:
-            one(mode, lps, ctas)                          # settle into this schedule
-            t0, t1 = ev(), ev()
-            t0.record(main)
-            w0 = time.time()
-            for _ in range(reps):
-                one(mode, lps, ctas)
-            t1.record(main)
-            torch.cuda.synchronize()
-            times[name].append(t0.elapsed_time(t1) / reps)
-            clocks[name].append(sampler.summary(w0 + 0.3, time.time()))
+            if name == "compute_only":
+                continue
+            t, clk = block(mode, lps, ctas)
+            after, _ = block("compute", 1, 0)
+            times[name].append(t)
+            clocks[name].append(clk)
+            times["compute_only"].append(after)
+            exposed[name].append(t - (before + after) / 2)
+            before = after
     time.sleep(0.1)
     sampler.stop()
     res = {name: round(statistics.mean(v), 3) for name, v in times.items()}
-    comp = res["compute_only"]
-    best_lw = min((k for k in res if k.startswith("layerwise")), key=lambda k: res[k])
-    line = {"metric": METRIC + " (layer-wise retrieval pipelined with prefill compute)",
+    exp_ms = {k: round(statistics.mean(v), 3) for k, v in exposed.items()}
+    best_lw = min((k for k in exp_ms if k.startswith("layerwise")), key=lambda k: exp_ms[k])
+    store_gbs = []
+    for _ in range(3):
+        t0, t1 = ev(), ev()
+        t0.record(side)
+        kvs.kvs_store(g, buf.plane_ptrs, w.num_blocks, buf.store_requests, side, 0)
+        t1.record(side)
+        torch.cuda.synchronize()
+        store_gbs.append(suffix * token_bytes(g) / (t0.elapsed_time(t1) / 1e3) / 1e9)
+    line = {"metric": METRIC + " (layer-wise retrieval and store-back pipelined with prefill compute)",
             "unit": "ms per prefill", "higher_is_better": False,
             "config": {"workload": describe(w), "compute": f"per layer one bf16 GEMM {M}x{K}x{N} "
                        "(Llama-3-8B q/k/v/o/MLP widths over the uncached suffix tokens)",
+                       "store": f"the {suffix}-token computed suffix to pinned host chunks",
                        "retrieval_stream_priority": args.side_priority,
-                       "timing": f"{reps} back-to-back prefills per schedule, two interleaved passes, mean"},
+                       "timing": f"{reps} back-to-back prefills per schedule, each schedule bracketed by "
+                                 "compute-only blocks, two passes, mean"},
             "ms_per_prefill": res,
-            "per_pass_ms": {k: [round(x, 3) for x in v] for k, v in times.items()},
+            "exposed_copy_ms": exp_ms,
+            "exposed_copy_ms_per_pass": {k: [round(x, 3) for x in v] for k, v in exposed.items()},
             "retrieve_alone_ms": round(min(retrieve_alone), 3),
             "retrieval_gbs_alone": round(buf.payload_bytes / (min(retrieve_alone) / 1e3) / 1e9, 2),
-            "exposed_retrieval_ms": {k: round(v - comp, 3) for k, v in res.items() if k != "compute_only"},
+            "store_alone_gbs": round(max(store_gbs), 2),
             "best_layerwise": best_lw,
             "speedup_vs_serial": round(res["serial"] / res[best_lw], 4),
             "clocks": {k: v[-1] for k, v in clocks.items()}}

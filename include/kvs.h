@@ -191,12 +191,20 @@ int kvs_retrieve_layers(const kvs_geometry* geom, const kvs_paged_cache* cache,
                         int32_t layers_per_step, void* const* layer_events,
                         void* cuda_stream, uint32_t flags);
 
-/* Layer-wise store-back: kvs_store in layer groups, recording layer_events[k]
- * after group k (for storing KV while later layers are still being computed). */
+/* Layer-wise store-back: kvs_store in layer groups, so that newly computed KV
+ * leaves the GPU while later layers are still being computed.  Before group k
+ * (layers [k * layers_per_step, (k + 1) * layers_per_step)) is copied,
+ * cuda_stream waits on ready_events[k] (cudaStreamWaitEvent: the caller
+ * records it on its compute stream once those layers' KV is in the cache,
+ * before this call); after group k, layer_events[k] is recorded.  Either array
+ * may be NULL, and so may any of its entries (no wait / no record).  Groups are
+ * always separate launches here.  KVS_F_FORCE_HBMCOPY returns
+ * KVS_ERR_UNSUPPORTED; KVS_F_LAYER_SIGNAL together with ready_events is
+ * KVS_ERR_INVALID_ARG (a resident launch cannot wait between groups). */
 int kvs_store_layers(const kvs_geometry* geom, const kvs_paged_cache* cache,
                      const kvs_request* requests, int32_t num_requests,
-                     int32_t layers_per_step, void* const* layer_events,
-                     void* cuda_stream, uint32_t flags);
+                     int32_t layers_per_step, void* const* ready_events,
+                     void* const* layer_events, void* cuda_stream, uint32_t flags);
 
 /* Bandwidths measured by kvs_query_bw, in GB/s (1e9 bytes per second). */
 typedef struct kvs_bw_report {
@@ -395,7 +403,7 @@ void* kvs_tier_slot(const kvs_tier* tier, int64_t slot);
 
 /* ABI version of this header: major * 10000 + minor * 100 + patch. */
 int kvs_version(void);
-#define KVS_VERSION 10400
+#define KVS_VERSION 10500
 
 #ifdef __cplusplus
 }

@@ -584,13 +584,16 @@ int read_error_word(DevState& st, cudaStream_t s) {
 // caller's stream.
 int copy_call(const kvs_geometry* g, const kvs_paged_cache* cache, const kvs_request* reqs,
               int32_t nreq, void* stream, uint32_t flags, bool retrieve,
-              int32_t layers_per_step = 0, void* const* layer_events = nullptr) {
+              int32_t layers_per_step = 0, void* const* layer_events = nullptr,
+              void* const* ready_events = nullptr) {
     const bool f_host = flags & KVS_F_FORCE_HOSTLINK, f_hbm = flags & KVS_F_FORCE_HBMCOPY;
     const bool f_ldg = flags & KVS_F_FORCE_LDG, f_tma = flags & KVS_F_FORCE_TMA;
     if ((f_host && f_hbm) || (f_ldg && f_tma))
         return fail(KVS_ERR_INVALID_ARG, "conflicting FORCE flags");
     if ((flags & KVS_F_LAYER_LAUNCHES) && (flags & KVS_F_LAYER_SIGNAL))
         return fail(KVS_ERR_INVALID_ARG, "KVS_F_LAYER_LAUNCHES and KVS_F_LAYER_SIGNAL together");
+    if (ready_events && (flags & KVS_F_LAYER_SIGNAL))
+        return fail(KVS_ERR_INVALID_ARG, "ready events need one launch per group, not KVS_F_LAYER_SIGNAL");
     if (layers_per_step < 0) return fail(KVS_ERR_INVALID_ARG, "layers_per_step must be positive");
     if (layers_per_step > 0 && f_hbm)
         return fail(KVS_ERR_UNSUPPORTED, "layer-wise copies move host chunks over the host link only");
@@ -695,6 +698,8 @@ int copy_call(const kvs_geometry* g, const kvs_paged_cache* cache, const kvs_req
     for (int k = 0; k < groups; ++k) {
         const uint32_t p0 = (uint32_t)(2 * k * lps);
         const uint32_t np = (uint32_t)(2 * (std::min(L, (k + 1) * lps) - k * lps));
+        if (ready_events && ready_events[k])
+            KVS_CUDA(cudaStreamWaitEvent(s, (cudaEvent_t)ready_events[k], 0));
         if (fork) {
             KVS_CUDA(cudaEventRecord(st.ev_aux_fork, s));
             KVS_CUDA(cudaStreamWaitEvent(st.aux_stream, st.ev_aux_fork, 0));
@@ -916,12 +921,13 @@ int kvs_retrieve_layers(const kvs_geometry* geom, const kvs_paged_cache* cache, 
 }
 
 int kvs_store_layers(const kvs_geometry* geom, const kvs_paged_cache* cache, const kvs_request* requests,
-                     int32_t num_requests, int32_t layers_per_step, void* const* layer_events,
-                     void* cuda_stream, uint32_t flags) {
+                     int32_t num_requests, int32_t layers_per_step, void* const* ready_events,
+                     void* const* layer_events, void* cuda_stream, uint32_t flags) {
     std::lock_guard<std::mutex> lk(g_mu);
     t_error.clear();
     if (layers_per_step <= 0) return fail(KVS_ERR_INVALID_ARG, "layers_per_step must be positive");
-    return copy_call(geom, cache, requests, num_requests, cuda_stream, flags, false, layers_per_step, layer_events);
+    return copy_call(geom, cache, requests, num_requests, cuda_stream, flags, false, layers_per_step, layer_events,
+                     ready_events);
 }
 
 int kvs_query_bw(kvs_bw_report* out, void* cuda_stream, int64_t probe_bytes) {

@@ -156,12 +156,15 @@ def lib():
                 fn.argtypes = [ctypes.POINTER(kvs_geometry), ctypes.POINTER(kvs_paged_cache),
                                ctypes.POINTER(kvs_request), ctypes.c_int32, P, ctypes.c_uint32]
                 fn.restype = ctypes.c_int
-            for name in ("kvs_retrieve_layers", "kvs_store_layers"):
-                fn = getattr(L, name)
-                fn.argtypes = [ctypes.POINTER(kvs_geometry), ctypes.POINTER(kvs_paged_cache),
-                               ctypes.POINTER(kvs_request), ctypes.c_int32, ctypes.c_int32,
-                               ctypes.POINTER(ctypes.c_void_p), P, ctypes.c_uint32]
-                fn.restype = ctypes.c_int
+            EVP = ctypes.POINTER(ctypes.c_void_p)
+            L.kvs_retrieve_layers.argtypes = [ctypes.POINTER(kvs_geometry), ctypes.POINTER(kvs_paged_cache),
+                                              ctypes.POINTER(kvs_request), ctypes.c_int32, ctypes.c_int32,
+                                              EVP, P, ctypes.c_uint32]
+            L.kvs_retrieve_layers.restype = ctypes.c_int
+            L.kvs_store_layers.argtypes = [ctypes.POINTER(kvs_geometry), ctypes.POINTER(kvs_paged_cache),
+                                           ctypes.POINTER(kvs_request), ctypes.c_int32, ctypes.c_int32,
+                                           EVP, EVP, P, ctypes.c_uint32]
+            L.kvs_store_layers.restype = ctypes.c_int
             U64P, I64P, I32P = (ctypes.POINTER(ctypes.c_uint64), ctypes.POINTER(ctypes.c_int64),
                                 ctypes.POINTER(ctypes.c_int32))
             tier_sigs = {
@@ -343,14 +346,26 @@ def kvs_retrieve_layers(geom, planes, num_blocks, requests, layers_per_step, lay
                                             int(layers_per_step), ev, _stream(stream), ctypes.c_uint32(flags)))
 
 
+def _wait_events(events):
+    """cudaEvent_t handles of events to wait on; an event never recorded (no handle yet)
+    has nothing to wait for and is passed as NULL."""
+    if events is None:
+        return None, None
+    handles = [0 if e is None else int(e.cuda_event) if hasattr(e, "cuda_event") else int(e) for e in events]
+    arr = (ctypes.c_void_p * max(1, len(handles)))(*handles)
+    return arr, ctypes.cast(arr, ctypes.POINTER(ctypes.c_void_p))
+
+
 def kvs_store_layers(geom, planes, num_blocks, requests, layers_per_step, layer_events=None,
-                     stream=None, flags: int = 0) -> int:
-    """Layer-wise :func:`kvs_store`."""
+                     stream=None, flags: int = 0, ready_events=None) -> int:
+    """Layer-wise :func:`kvs_store`: group k waits on ``ready_events[k]`` (recorded by the
+    caller once those layers' KV is computed) and records ``layer_events[k]`` when copied."""
     g = _geometry(geom)
     m = _Marshalled(planes, num_blocks, requests)
+    keep_r, rev = _wait_events(ready_events)
     keep, ev = _events(layer_events, stream)
     return _check(lib().kvs_store_layers(ctypes.byref(g), ctypes.byref(m.cache), m.reqs, m.n,
-                                         int(layers_per_step), ev, _stream(stream), ctypes.c_uint32(flags)))
+                                         int(layers_per_step), rev, ev, _stream(stream), ctypes.c_uint32(flags)))
 
 
 def kvs_query_bw(stream=None, probe_bytes: int = 0) -> dict:

@@ -25,7 +25,7 @@ def test_library_exports_every_declared_function():
     for n in names:
         assert hasattr(lib, n), n
     assert set(names) == set(kvs.EXPORTED)
-    assert kvs.kvs_version() == 10400
+    assert kvs.kvs_version() == 10500
 
 
 def test_struct_layouts_match_header():
@@ -108,6 +108,10 @@ def test_layerwise_argument_checks(fn):
     with pytest.raises(kvs.KvsError) as ei:
         fn(G, [FAKE] * 4, 8, [_req()], 1, None, None, kvs.KVS_F_LAYER_LAUNCHES | kvs.KVS_F_LAYER_SIGNAL)
     assert ei.value.code == kvs.KVS_ERR_INVALID_ARG
+    if fn is kvs.kvs_store_layers:
+        with pytest.raises(kvs.KvsError) as ei:
+            fn(G, [FAKE] * 4, 8, [_req()], 1, None, None, kvs.KVS_F_LAYER_SIGNAL, ready_events=[None, None])
+        assert ei.value.code == kvs.KVS_ERR_INVALID_ARG
     with pytest.raises(kvs.KvsError) as ei:
         fn(G, [FAKE] * 4, 8, [_req(table=(0, 1, 9, 3))], 1)
     assert ei.value.code == kvs.KVS_ERR_BOUNDS

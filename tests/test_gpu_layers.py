@@ -87,6 +87,39 @@ def test_store_layers_matches_oracle(lps):
     gc.check_store(buf)
 
 
+@pytest.mark.parametrize("lps", [1, 2])
+def test_store_layers_waits_for_each_groups_ready_event(lps):
+    """A producer stream rewrites layer group k's planes after a delay, then records
+    ready[k]; the store must copy the rewritten bytes of every group (a store that did
+    not wait would copy the planes' earlier contents)."""
+    w = synth.custom(4, 8, 128, 16, 256, 128, [1024, 700], [0, 0], seed=11, store_tokens=[768, 700])
+    g = w.geom
+    buf = buffers.allocate(w, store=True, plane_init="random")
+    groups = -(-g.layers // lps)
+    gen = torch.Generator(device="cuda").manual_seed(3)
+    fresh = torch.randint(-32768, 32767, tuple(buf.planes.shape), dtype=torch.int16, device="cuda", generator=gen)
+    producer, copier = torch.cuda.Stream(), torch.cuda.Stream()
+    ready = [torch.cuda.Event() for _ in range(groups)]
+    torch.cuda.synchronize()
+    with torch.cuda.stream(producer):
+        for k in range(groups):
+            torch.cuda._sleep(20_000_000)                 # ~10 ms: long after an unblocked copy
+            p0, p1 = 2 * k * lps, 2 * min(g.layers, (k + 1) * lps)
+            buf.planes[p0:p1].copy_(fresh[p0:p1])
+            ready[k].record(producer)
+    kvs.kvs_store_layers(g, buf.plane_ptrs, w.num_blocks, buf.store_requests, lps, None, copier,
+                         kvs.KVS_F_VALIDATE, ready_events=ready)
+    torch.cuda.synchronize()
+    planes_np = [fresh[p].cpu().numpy().view(np.uint16) for p in range(2 * g.layers)]
+    fill = synth.sentinel(2)
+    for r, req in enumerate(buf.store_requests):
+        want = [np.full(t.numel(), fill, dtype=np.uint16) for t in buf.store_chunks[r]]
+        assert oracle.store(g.layers, g.kv_heads, g.head_dim, g.block_size, planes_np, w.num_blocks,
+                            req.first_token, want, req.block_table) == 0
+        for j, (t, e) in enumerate(zip(buf.store_chunks[r], want)):
+            assert np.array_equal(t.cpu().numpy().view(np.uint16), e), (lps, r, j)
+
+
 def test_empty_layerwise_call_still_records_events():
     w = _workload()
     buf = buffers.allocate(w)
