@@ -643,25 +643,33 @@ def run_overlap(args):
         done = [t for t in (g0.elapsed_time(e) for e in gev) if t <= window_ms]
         return (2 * 8192 ** 3 * len(done) / (done[-1] / 1e3) / 1e12) if done else float("nan")
 
+    def copy(reqs, flags):
+        """One retrieval of ``reqs``; KVS_F_LAYER_LAUNCHES here means one launch per layer
+        (a layer-wise call without events), which hands SMs back between layers."""
+        if flags & kvs.KVS_F_LAYER_LAUNCHES:
+            kvs.kvs_retrieve_layers(g, ptrs, w.num_blocks, reqs, 1, None, side, flags)
+        else:
+            kvs.kvs_retrieve(g, ptrs, w.num_blocks, reqs, side, flags)
+
     def retrieval(flags, with_gemm):
         total_ms, gemm_n, gemm_during, gemm_alone = 0.0, 0, [], []
         for k in range(passes):
             if k:
                 pinned.copy_(refill_src)                 # refill between passes (untimed)
             reqs = pass_requests(k)
-            kvs.kvs_retrieve(g, ptrs, w.num_blocks, reqs, side, flags)   # warm
+            copy(reqs, flags)                            # warm
             torch.cuda.synchronize()
             if not with_gemm:
                 r0, r1 = ev(), ev()
                 r0.record(side)
-                kvs.kvs_retrieve(g, ptrs, w.num_blocks, reqs, side, flags)
+                copy(reqs, flags)
                 r1.record(side)
                 torch.cuda.synchronize()
                 total_ms += r0.elapsed_time(r1)
                 continue
             # GEMMs queued so that they outlast the retrieval
             iters = int(1.3 * (tokens_pass * per_tok * 2 / (host_peak * 1e9)) / (gemm_ms / 1e3)) + 4
-            g0, gev, r1 = gemm_window(iters, lambda: kvs.kvs_retrieve(g, ptrs, w.num_blocks, reqs, side, flags))
+            g0, gev, r1 = gemm_window(iters, lambda: copy(reqs, flags))
             r_ms = g0.elapsed_time(r1)
             total_ms += r_ms
             gemm_during.append(rate_within(g0, gev, r_ms))
@@ -680,7 +688,9 @@ def run_overlap(args):
                 ("hostlink_8ctas", kvs.KVS_F_FORCE_HOSTLINK | kvs.KVS_F_MAX_CTAS(8)),
                 ("hostlink_12ctas", kvs.KVS_F_FORCE_HOSTLINK | kvs.KVS_F_MAX_CTAS(12)),
                 ("hostlink_24ctas", kvs.KVS_F_FORCE_HOSTLINK | kvs.KVS_F_MAX_CTAS(24)),
-                ("hbmcopy", kvs.KVS_F_FORCE_HBMCOPY)]
+                ("hbmcopy", kvs.KVS_F_FORCE_HBMCOPY),
+                ("layer_launches", kvs.KVS_F_LAYER_LAUNCHES),
+                ("layer_launches_96ctas", kvs.KVS_F_LAYER_LAUNCHES | kvs.KVS_F_MAX_CTAS(96))]
     for name, fl in variants:
         results[name] = {"alone": retrieval(fl, False), "with_gemm": retrieval(fl, True)}
     line = {"metric": METRIC + " (overlap with a bf16 GEMM loop)", "unit": "GB/s",
