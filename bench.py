@@ -53,6 +53,8 @@ def parse_args(argv=None):
                     help="llama8b: layer-wise retrieval pipelined with a per-layer prefill GEMM")
     ap.add_argument("--tempokv", action="store_true",
                     help="TempoKV control-plane model driven by the retrieval rate measured in this run")
+    ap.add_argument("--duplex", action="store_true",
+                    help="llama8b: retrieval (host->GPU) and store-back (GPU->host) at the same time")
     ap.add_argument("--side-priority", choices=["normal", "high"], default="high",
                     help="priority of the retrieval stream in --overlap runs")
     return ap.parse_args(argv)
@@ -920,6 +922,97 @@ def run_tempokv(args):
     return 0
 
 
+def run_duplex(args):
+    """Retrieval of the matched prefix and store-back of the computed suffix (4 GiB each,
+    pinned host chunks) on two streams at once, against each alone: how much of the two
+    host-link directions can be used together."""
+    import torch
+    from paper_2609_35065_gb300 import buffers, kvs
+
+    torch.cuda.set_device(0)
+    kvs.lib()
+    s1, s2 = torch.cuda.Stream(), torch.cuda.Stream()
+    bw = kvs.kvs_query_bw(s1, 1 << 30)
+    w = workload(args.config)
+    g = w.geom
+    for r in w.requests:
+        r.store_tokens = r.prompt_tokens - r.matched_tokens
+    buf = buffers.allocate(w, store=True)
+    rbytes = buf.payload_bytes
+    sbytes = sum(r.store_tokens for r in w.requests) * token_bytes(g)
+
+    def ev():
+        return torch.cuda.Event(enable_timing=True)
+
+    def run(retrieve, store, caps):
+        torch.cuda.synchronize()
+        t0 = ev()
+        t0.record(s1)
+        s2.wait_event(t0)
+        if retrieve:
+            kvs.kvs_retrieve(g, buf.plane_ptrs, w.num_blocks, buf.requests, s1, kvs.KVS_F_MAX_CTAS(caps[0]))
+        if store:
+            kvs.kvs_store(g, buf.plane_ptrs, w.num_blocks, buf.store_requests, s2, kvs.KVS_F_MAX_CTAS(caps[1]))
+        e1, e2 = ev(), ev()
+        e1.record(s1)
+        e2.record(s2)
+        torch.cuda.synchronize()
+        return t0.elapsed_time(e1), t0.elapsed_time(e2)
+
+    reps = max(3, min(args.steps, 10))
+    res = {}
+    for name, r, st, caps in (("retrieve_alone", True, False, (0, 0)), ("store_alone", False, True, (0, 0)),
+                              ("both_default_caps", True, True, (0, 0)), ("both_64_64", True, True, (64, 64)),
+                              ("both_96_96", True, True, (96, 96))):
+        run(r, st, caps)
+        ts = [run(r, st, caps) for _ in range(reps)]
+        r_ms = statistics.median(t[0] for t in ts)
+        s_ms = statistics.median(t[1] for t in ts)
+        d = {}
+        if r:
+            d["retrieve_gbs"] = round(rbytes / r_ms / 1e6, 2)
+        if st:
+            d["store_gbs"] = round(sbytes / s_ms / 1e6, 2)
+        if r and st:
+            d["aggregate_gbs"] = round((rbytes + sbytes) / max(r_ms, s_ms) / 1e6, 2)
+        res[name] = d
+    # the copy engines in both directions at once (1 GiB each way, pinned host memory)
+    n = 1 << 30
+    h_in = torch.empty(n, dtype=torch.uint8, pin_memory=True)
+    h_out = torch.empty(n, dtype=torch.uint8, pin_memory=True)
+    d_in = torch.empty(n, dtype=torch.uint8, device="cuda")
+    d_out = torch.zeros(n, dtype=torch.uint8, device="cuda")
+    ce = {}
+    for name, h2d, d2h in (("h2d_alone", True, False), ("d2h_alone", False, True), ("both", True, True)):
+        ts = []
+        for _ in range(reps + 1):
+            torch.cuda.synchronize()
+            t0 = ev()
+            t0.record(s1)
+            s2.wait_event(t0)
+            if h2d:
+                with torch.cuda.stream(s1):
+                    d_in.copy_(h_in, non_blocking=True)
+            if d2h:
+                with torch.cuda.stream(s2):
+                    h_out.copy_(d_out, non_blocking=True)
+            e1, e2 = ev(), ev()
+            e1.record(s1)
+            e2.record(s2)
+            torch.cuda.synchronize()
+            ts.append(max(t0.elapsed_time(e1) if h2d else 0.0, t0.elapsed_time(e2) if d2h else 0.0))
+        ce[name] = round((n * (h2d + d2h)) / statistics.median(ts[1:]) / 1e6, 2)
+    res["copy_engines_gbs"] = ce
+    line = {"metric": METRIC + " (retrieval and store-back concurrently)", "unit": "GB/s",
+            "config": {"workload": describe(w), "store": "computed suffix to pinned host chunks",
+                       "timing": f"median of {reps} runs"},
+            "host_link_probe": {"h2d_gbs": round(bw["h2d_copy_engine_gbs"], 2),
+                                "d2h_gbs": round(bw["d2h_copy_engine_gbs"], 2)},
+            "hostlink_ctas": bw["hostlink_ctas"], "store_ctas": bw["store_ctas"], **res}
+    print(json.dumps(line), flush=True)
+    return 0
+
+
 def main(argv=None):
     args = parse_args(argv)
     if args.tempokv:
@@ -930,6 +1023,8 @@ def main(argv=None):
         return run_overlap(args)
     if args.layerwise:
         return run_layerwise(args)
+    if args.duplex:
+        return run_duplex(args)
     return run_ours(args)
 
 
