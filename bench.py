@@ -53,6 +53,8 @@ def parse_args(argv=None):
                     help="llama8b: layer-wise retrieval pipelined with a per-layer prefill GEMM")
     ap.add_argument("--tempokv", action="store_true",
                     help="TempoKV control-plane model driven by the retrieval rate measured in this run")
+    ap.add_argument("--sizes", action="store_true",
+                    help="llama8b shape: retrieval rate against call size (1 to 128 chunks)")
     ap.add_argument("--duplex", action="store_true",
                     help="llama8b: retrieval (host->GPU) and store-back (GPU->host) at the same time")
     ap.add_argument("--side-priority", choices=["normal", "high"], default="high",
@@ -1013,6 +1015,76 @@ def run_duplex(args):
     return 0
 
 
+def run_sizes(args):
+    """Retrieval rate against call size, host and HBM sources: the GPU time of back-to-back
+    calls (CUDA events) and the latency of one synchronous call through the API
+    (marshalling, planning, upload, launch, completion), for 1 to 128 chunks of 32 MiB."""
+    import torch
+    from paper_2609_35065_gb300 import buffers, kvs
+
+    torch.cuda.set_device(0)
+    kvs.lib()
+    stream = torch.cuda.Stream()
+    kvs.kvs_query_bw(stream, 1 << 30)
+    w = workload("llama8b")
+    g = w.geom
+    buf = buffers.allocate(w)
+    per_tok = 2 * g.layers * g.row_elems
+    dpool = torch.empty_like(buf.host_pool, device="cuda")
+    dpool.copy_(buf.host_pool)
+    chunk_bytes = g.chunk_tokens * token_bytes(g)
+
+    def requests(n, device):
+        out, at, left = [], 0, n
+        for r in buf.requests:
+            if left == 0:
+                break
+            cs = []
+            for c in r.chunks[:left]:
+                base = dpool[at:at + c.num_tokens * per_tok] if device else c.base
+                cs.append(kvs.ChunkArg(base, c.num_tokens, kvs.KVS_SRC_DEVICE if device else c.residency))
+                at += c.num_tokens * per_tok
+            at += sum(c.num_tokens for c in r.chunks[left:]) * per_tok
+            left -= len(cs)
+            out.append(kvs.RequestArg(r.block_table, cs, r.first_token))
+        return out
+
+    reps = max(5, min(args.steps, 20))
+    res = {}
+    for source in ("host", "device"):
+        rows = {}
+        for n in (1, 2, 4, 8, 16, 32, 64, 128):
+            reqs = requests(n, source == "device")
+            for _ in range(3):
+                kvs.kvs_retrieve(g, buf.plane_ptrs, w.num_blocks, reqs, stream, 0)
+            torch.cuda.synchronize()
+            t0, t1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+            t0.record(stream)
+            for _ in range(reps):
+                kvs.kvs_retrieve(g, buf.plane_ptrs, w.num_blocks, reqs, stream, 0)
+            t1.record(stream)
+            torch.cuda.synchronize()
+            gpu_ms = t0.elapsed_time(t1) / reps
+            lat = []
+            for _ in range(reps):
+                h0 = time.perf_counter()
+                kvs.kvs_retrieve(g, buf.plane_ptrs, w.num_blocks, reqs, stream, 0)
+                stream.synchronize()
+                lat.append((time.perf_counter() - h0) * 1e3)
+            nbytes = n * chunk_bytes
+            lat_ms = statistics.median(lat)
+            rows[str(n)] = {"bytes": nbytes, "gpu_ms": round(gpu_ms, 4), "gpu_gbs": round(nbytes / gpu_ms / 1e6, 1),
+                            "call_latency_ms": round(lat_ms, 4), "latency_gbs": round(nbytes / lat_ms / 1e6, 1)}
+        res[source] = rows
+    line = {"metric": METRIC + " (call size sweep)", "unit": "GB/s",
+            "config": {"workload": "llama8b geometry, 1-128 chunks of 256 tokens (32 MiB each)",
+                       "timing": f"gpu: {reps} back-to-back calls, CUDA events; latency: median of {reps} "
+                                 "synchronous calls through the Python API"},
+            **res}
+    print(json.dumps(line), flush=True)
+    return 0
+
+
 def main(argv=None):
     args = parse_args(argv)
     if args.tempokv:
@@ -1025,6 +1097,8 @@ def main(argv=None):
         return run_layerwise(args)
     if args.duplex:
         return run_duplex(args)
+    if args.sizes:
+        return run_sizes(args)
     return run_ours(args)
 
 

@@ -62,9 +62,17 @@ class Buffers:
     plane_init: str = "sentinel"
     notes: dict = field(default_factory=dict)
 
+    _ptrs: tuple = (None, None)                    # (planes base address, plane addresses)
+
     @property
     def plane_ptrs(self) -> list[int]:
-        return [int(self.planes[p].data_ptr()) for p in range(self.planes.shape[0])]
+        """Addresses of the 2L planes (rows of one contiguous tensor), computed once per
+        planes tensor: a call site that passes them every step pays nothing for it."""
+        base = int(self.planes.data_ptr())
+        if self._ptrs[0] != base:
+            row = self.planes.stride(0) * self.planes.element_size()
+            self._ptrs = (base, [base + p * row for p in range(self.planes.shape[0])])
+        return self._ptrs[1]
 
     @property
     def payload_bytes(self) -> int:

@@ -208,12 +208,15 @@ def lib():
 
 # ---- marshalling helpers --------------------------------------------------
 def _addr(x) -> int:
+    if type(x) is int:
+        return x
+    ptr = getattr(x, "data_ptr", None)
+    if ptr is not None:
+        return int(ptr())
     if x is None:
         return 0
     if isinstance(x, int):
         return x
-    if hasattr(x, "data_ptr"):
-        return int(x.data_ptr())
     if isinstance(x, np.ndarray):
         return int(x.ctypes.data)
     raise TypeError(f"cannot take the address of {type(x)!r}")
@@ -263,7 +266,10 @@ class _Marshalled:
     """The C call's argument arrays (kept alive for the duration of one call)."""
 
     def __init__(self, planes, num_blocks, requests):
-        self.planes = np.array([_addr(p) for p in planes] or [0], dtype=np.uint64)
+        if planes and all(type(p) is int for p in planes):
+            self.planes = np.array(planes, dtype=np.uint64)
+        else:
+            self.planes = np.array([_addr(p) for p in planes] or [0], dtype=np.uint64)
         self.cache = kvs_paged_cache(ctypes.cast(int(self.planes.ctypes.data), ctypes.POINTER(ctypes.c_void_p)),
                                      int(num_blocks))
         counts = [len(r.chunks) for r in requests]
@@ -277,11 +283,14 @@ class _Marshalled:
         self.tables = [np.ascontiguousarray(r.block_table, dtype=np.int32) for r in requests]
         reqs = np.zeros(max(1, len(requests)), dtype=_REQ_DT)
         if requests:
-            starts = np.concatenate([[0], np.cumsum(counts)[:-1]]).astype(np.uint64)
+            base, step, at, starts = chunks.ctypes.data, _CHUNK_DT.itemsize, 0, []
+            for n in counts:                          # address of each request's first chunk
+                starts.append(base + at * step)
+                at += n
             reqs["first_token"] = [r.first_token for r in requests]
             reqs["num_tokens"] = [sum(c.num_tokens for c in r.chunks) if r.num_tokens is None else r.num_tokens
                                   for r in requests]
-            reqs["chunks"] = np.uint64(chunks.ctypes.data) + starts * np.uint64(_CHUNK_DT.itemsize)
+            reqs["chunks"] = starts
             reqs["num_chunks"] = counts
             reqs["block_table_len"] = [t.size for t in self.tables]
             reqs["block_table"] = [t.ctypes.data for t in self.tables]
