@@ -36,6 +36,38 @@ def test_llama8b_host_source(flags):
     gc.free(buf)
 
 
+def test_llama8b_in_the_bench_launch_configuration():
+    """The calls bench.py times: after kvs_query_bw has chosen the variants and the
+    host-link grid, flags 0 on a side stream (no validation pass), the host-source
+    batch and then the same chunks staged in HBM; every element checked."""
+    s = torch.cuda.Stream()
+    choice = kvs.kvs_query_bw(s, 1 << 30)
+    buf = buffers.allocate(synth.llama8b())
+    w = buf.workload
+    kvs.kvs_retrieve(w.geom, buf.plane_ptrs, w.num_blocks, buf.requests, s, 0)
+    s.synchronize()
+    assert kvs.kvs_check_errors(s) == kvs.KVS_OK
+    gc.check_retrieve(buf)
+    # the same batch from an HBM staging copy of the chunks, into sentinel planes
+    dpool = buf.host_pool.to("cuda")
+    per_tok = 2 * w.geom.layers * w.geom.row_elems
+    dreqs, at = [], 0
+    for r in buf.requests:
+        cs = []
+        for c in r.chunks:
+            cs.append(kvs.ChunkArg(dpool[at:at + c.num_tokens * per_tok], c.num_tokens, kvs.KVS_SRC_DEVICE))
+            at += c.num_tokens * per_tok
+        dreqs.append(kvs.RequestArg(r.block_table, cs, r.first_token))
+    buf.planes.fill_(np.array([synth.SENTINEL_BF16], dtype=np.uint16).view(np.int16)[0].item())
+    kvs.kvs_retrieve(w.geom, buf.plane_ptrs, w.num_blocks, dreqs, s, 0)
+    s.synchronize()
+    assert kvs.kvs_check_errors(s) == kvs.KVS_OK
+    gc.check_retrieve(buf)
+    assert choice["chosen_kernel_device"] in (kvs.KVS_KERNEL_LDG, kvs.KVS_KERNEL_TMA)
+    del dpool
+    gc.free(buf)
+
+
 @pytest.mark.parametrize("ratio,flags", [(25, 0), (50, 0), (75, 0), (50, kvs.KVS_F_FORCE_TMA),
                                          (50, kvs.KVS_F_FORCE_LDG)],
                          ids=["25", "50", "75", "50_tma", "50_ldg"])
