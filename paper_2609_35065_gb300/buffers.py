@@ -175,5 +175,8 @@ def allocate(w: synth.Workload, device: str = "cuda", store: bool = False,
             store_chunks.append(mine)
             store_requests.append(RequestArg(r.block_table, [ChunkArg(t, t.numel() // per_tok, res) for t in mine],
                                              first_token=r.store_start if r.store_tokens else 0))
+    if torch.device(device).type == "cuda":
+        # the fills ran on torch's stream; copies issued next on other streams must see them
+        torch.cuda.synchronize()
     return Buffers(w, planes, chunks, store_chunks, requests, store_requests,
                    host_pool, device_pool, store_pool, plane_init)

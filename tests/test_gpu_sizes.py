@@ -59,6 +59,7 @@ def test_llama8b_in_the_bench_launch_configuration():
             at += c.num_tokens * per_tok
         dreqs.append(kvs.RequestArg(r.block_table, cs, r.first_token))
     buf.planes.fill_(np.array([synth.SENTINEL_BF16], dtype=np.uint16).view(np.int16)[0].item())
+    s.wait_stream(torch.cuda.current_stream())          # the refill runs on torch's stream
     kvs.kvs_retrieve(w.geom, buf.plane_ptrs, w.num_blocks, dreqs, s, 0)
     s.synchronize()
     assert kvs.kvs_check_errors(s) == kvs.KVS_OK
