@@ -248,6 +248,20 @@ int kvs_get_choice(kvs_bw_report* out);
  */
 int kvs_check_errors(void* cuda_stream);
 
+/*
+ * Pipelined form of kvs_check_errors for loops that keep the GPU busy: enqueues
+ * on cuda_stream a copy of this device's error word into *host_word followed by
+ * a reset of the word, and returns at once without synchronising.  host_word
+ * must be page-locked host memory owned by the caller and stay valid until the
+ * stream has passed the copy (record an event after this call and wait on it);
+ * it then holds 0 or the first KVS_ERR_* recorded by kernels that the stream ran
+ * before the copy.  Kernels of other streams of the same device that record an
+ * error between the copy and the reset are not reported; use one status stream
+ * per device.  Returns KVS_ERR_INVALID_ARG for a NULL host_word, KVS_ERR_CUDA if
+ * the copy cannot be enqueued.
+ */
+int kvs_enqueue_error_read(void* cuda_stream, int32_t* host_word);
+
 /* Message describing the last error on the calling thread ("" if none). */
 const char* kvs_last_error(void);
 
@@ -403,7 +417,7 @@ void* kvs_tier_slot(const kvs_tier* tier, int64_t slot);
 
 /* ABI version of this header: major * 10000 + minor * 100 + patch. */
 int kvs_version(void);
-#define KVS_VERSION 10500
+#define KVS_VERSION 10600
 
 #ifdef __cplusplus
 }

@@ -965,6 +965,19 @@ int kvs_check_errors(void* cuda_stream) {
     return read_error_word(*st, (cudaStream_t)cuda_stream);
 }
 
+int kvs_enqueue_error_read(void* cuda_stream, int32_t* host_word) {
+    std::lock_guard<std::mutex> lk(g_mu);
+    t_error.clear();
+    if (!host_word) return fail(KVS_ERR_INVALID_ARG, "host_word is NULL");
+    DevState* st = nullptr;
+    int rc = get_state(&st);
+    if (rc) return rc;
+    const cudaStream_t s = (cudaStream_t)cuda_stream;
+    KVS_CUDA(cudaMemcpyAsync(host_word, st->err, sizeof(int32_t), cudaMemcpyDeviceToHost, s));
+    KVS_CUDA(cudaMemsetAsync(st->err, 0, sizeof(int32_t), s));
+    return KVS_OK;
+}
+
 const char* kvs_last_error(void) { return t_error.c_str(); }
 
 int kvs_shutdown(void) {

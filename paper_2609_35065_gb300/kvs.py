@@ -56,6 +56,7 @@ KVS_KERNEL_LDG = 1
 KVS_KERNEL_TMA = 2
 
 EXPORTED = ("kvs_retrieve", "kvs_store", "kvs_query_bw", "kvs_get_choice", "kvs_check_errors",
+            "kvs_enqueue_error_read",
             "kvs_last_error", "kvs_shutdown", "kvs_version", "kvs_selftest_wait_timeout",
             "kvs_stat_launches", "kvs_retrieve_noalloc", "kvs_retrieve_layers", "kvs_store_layers",
             "kvs_tier_create", "kvs_tier_destroy", "kvs_tier_commit", "kvs_tier_staged",
@@ -192,6 +193,8 @@ def lib():
             L.kvs_get_choice.restype = ctypes.c_int
             L.kvs_check_errors.argtypes = [P]
             L.kvs_check_errors.restype = ctypes.c_int
+            L.kvs_enqueue_error_read.argtypes = [P, P]
+            L.kvs_enqueue_error_read.restype = ctypes.c_int
             L.kvs_last_error.argtypes = []
             L.kvs_last_error.restype = ctypes.c_char_p
             L.kvs_shutdown.argtypes = []
@@ -391,6 +394,12 @@ def kvs_get_choice() -> dict:
 
 def kvs_check_errors(stream=None) -> int:
     return _check(lib().kvs_check_errors(_stream(stream)))
+
+
+def kvs_enqueue_error_read(stream, host_word) -> int:
+    """Enqueue a copy of the device error word into ``host_word`` (a pinned int32 tensor
+    or address) and its reset, without synchronising; see kvs_check_errors."""
+    return _check(lib().kvs_enqueue_error_read(_stream(stream), ctypes.c_void_p(_addr(host_word))))
 
 
 def kvs_last_error() -> str:

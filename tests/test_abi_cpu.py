@@ -25,7 +25,7 @@ def test_library_exports_every_declared_function():
     for n in names:
         assert hasattr(lib, n), n
     assert set(names) == set(kvs.EXPORTED)
-    assert kvs.kvs_version() == 10500
+    assert kvs.kvs_version() == 10600
 
 
 def test_struct_layouts_match_header():

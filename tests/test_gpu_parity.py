@@ -53,6 +53,23 @@ def test_wait_timeout_selftest_then_context_usable():
     gc.check_retrieve(buf)
 
 
+def test_enqueue_error_read_does_not_synchronise():
+    """The status copy is queued behind the stream's work: the call returns while a
+    ~50 ms sleep kernel still runs ahead of it, and the word reads 0 once it has run."""
+    s = torch.cuda.Stream()
+    word = torch.full((1,), -7, dtype=torch.int32, pin_memory=True)
+    buf = buffers.allocate(synth.tiny(), store=True)
+    w = buf.workload
+    with torch.cuda.stream(s):
+        torch.cuda._sleep(100_000_000)
+    kvs.kvs_retrieve(w.geom, buf.plane_ptrs, w.num_blocks, buf.requests, s, 0)
+    assert kvs.kvs_enqueue_error_read(s, word) == kvs.KVS_OK
+    assert int(word[0]) == -7
+    s.synchronize()
+    assert int(word[0]) == kvs.KVS_OK
+    gc.check_retrieve(buf)
+
+
 @pytest.mark.parametrize("variant", sorted(VARIANTS))
 def test_tiny_retrieve_then_store_round_trip(variant):
     flags = VARIANTS[variant]
