@@ -116,3 +116,26 @@ def test_layerwise_argument_checks(fn):
         fn(G, [FAKE] * 4, 8, [_req(table=(0, 1, 9, 3))], 1)
     assert ei.value.code == kvs.KVS_ERR_BOUNDS
     assert fn(G, [FAKE] * 4, 8, [], 1) == kvs.KVS_OK          # nothing to copy, no events given
+
+
+def test_the_abi_from_plain_c(tmp_path):
+    """tests/c_abi_smoke.c, compiled as C99 against include/kvs.h and linked with
+    libkvs.so, runs its checks without a GPU."""
+    import os
+    import shutil
+    import subprocess
+    from paper_2609_35065_gb300 import build
+    gcc = shutil.which("gcc")
+    if gcc is None:
+        pytest.skip("no C compiler")
+    kvs.lib()                                               # builds the library if needed
+    here = os.path.dirname(os.path.abspath(__file__))
+    exe = str(tmp_path / "c_abi_smoke")
+    subprocess.run([gcc, "-std=c99", "-Wall", "-Wextra", "-Werror", "-pedantic",
+                    "-I", os.path.join(os.path.dirname(here), "include"),
+                    os.path.join(here, "c_abi_smoke.c"), build.LIB, "-o", exe,
+                    "-Wl,-rpath," + os.path.dirname(build.LIB)], check=True)
+    out = subprocess.run([exe], capture_output=True, text=True, timeout=60)
+    assert out.returncode == 0, (out.returncode, out.stderr)
+    assert out.stdout.strip() == "ok"
+
