@@ -58,7 +58,8 @@ extern "C" {
 #define KVS_ERR_BOUNDS      (-2)  /* block table shorter than the range, or a block id
                                      outside [0, num_blocks)                                */
 #define KVS_ERR_ALIAS       (-3)  /* one physical block named twice by one request, or
-                                     (KVS_F_VALIDATE) shared blocks with differing bytes   */
+                                     (KVS_F_VALIDATE) shared blocks with differing bytes,
+                                     or written memory overlapping written or read memory */
 #define KVS_ERR_CUDA        (-4)  /* a CUDA runtime call failed; see kvs_last_error()     */
 #define KVS_ERR_TIMEOUT     (-5)  /* a bounded device-side wait expired                    */
 #define KVS_ERR_NOMEM       (-6)  /* an internal buffer could not be allocated            */
@@ -73,7 +74,11 @@ extern "C" {
 /* ---- flags (bitwise OR) --------------------------------------------------- */
 #define KVS_F_VALIDATE       (1u << 0) /* synchronise the stream after the copy and return
                                           the device error word; also verify that blocks
-                                          shared by several requests receive equal bytes */
+                                          shared by several requests receive equal bytes,
+                                          that chunk pointers are what their residency
+                                          says, and (on the host, before any copy) that
+                                          the memory the call writes overlaps neither
+                                          itself nor the memory it reads              */
 #define KVS_F_FORCE_HOSTLINK (1u << 1) /* host chunks: SMs load/store host memory directly  */
 #define KVS_F_FORCE_HBMCOPY  (1u << 2) /* host chunks: copy engine to/from an HBM staging
                                           ring, SMs scatter/gather in HBM                    */

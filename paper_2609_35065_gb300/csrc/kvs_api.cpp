@@ -274,6 +274,56 @@ int validate_call(const kvs_geometry* g, const kvs_paged_cache* cache,
     return KVS_OK;
 }
 
+// With KVS_F_VALIDATE: the memory a call writes may overlap neither itself nor
+// the memory it reads (retrieve writes the planes and reads the chunks; store
+// writes the chunks and reads the planes), or the copy's result would depend
+// on the order of its stores.  Extents: a plane is num_blocks * B rows, a chunk
+// of n tokens 2L * n rows.  Sorted by start, a span overlaps an earlier one
+// exactly when some earlier span ends after it starts, so one sweep keeping
+// the furthest end (over all spans and over written spans) finds every
+// conflicting pair's later member.  Host only: no device work.
+int check_overlaps(const kvs_geometry* g, const kvs_paged_cache* cache, const kvs_request* reqs,
+                   int32_t nreq, bool retrieve) {
+    struct Span {
+        uint64_t lo, hi;
+        bool plane;
+        int32_t a, b;        // plane index, or (request, chunk)
+    };
+    const uint64_t row = (uint64_t)g->num_kv_heads * g->head_dim * g->elem_bytes;
+    const int P = 2 * g->num_layers;
+    std::vector<Span> sp;
+    sp.reserve(P);
+    for (int p = 0; p < P; ++p) {
+        const uint64_t lo = (uint64_t)cache->kv_planes[p];
+        sp.push_back({lo, lo + (uint64_t)cache->num_blocks * g->block_size * row, true, p, 0});
+    }
+    for (int32_t r = 0; r < nreq; ++r)
+        for (int32_t j = 0; j < reqs[r].num_chunks; ++j) {
+            const kvs_chunk& c = reqs[r].chunks[j];
+            const uint64_t lo = (uint64_t)c.base;
+            sp.push_back({lo, lo + (uint64_t)P * c.num_tokens * row, false, r, j});
+        }
+    std::sort(sp.begin(), sp.end(), [](const Span& x, const Span& y) { return x.lo < y.lo; });
+    auto name = [](const Span& x) {
+        char buf[64];
+        if (x.plane) snprintf(buf, sizeof buf, "plane %d", x.a);
+        else snprintf(buf, sizeof buf, "request %d chunk %d", x.a, x.b);
+        return std::string(buf);
+    };
+    const Span* far_all = nullptr;     // earlier span reaching furthest
+    const Span* far_written = nullptr; // same, among written spans
+    for (const Span& x : sp) {
+        const bool written = (x.plane == retrieve);
+        const Span* hit = written ? far_all : far_written;
+        if (hit && hit->hi > x.lo)
+            return fail(KVS_ERR_ALIAS, "%s overlaps %s (%s)", name(x).c_str(), name(*hit).c_str(),
+                        retrieve ? "retrieve writes planes" : "store writes chunks");
+        if (!far_all || x.hi > far_all->hi) far_all = &x;
+        if (written && (!far_written || x.hi > far_written->hi)) far_written = &x;
+    }
+    return KVS_OK;
+}
+
 // Second half: entries, block ids and de-duplication of shared physical blocks.
 int fill_plan(DevState& st, const kvs_geometry* g, const kvs_paged_cache* cache,
               const kvs_request* reqs, int32_t nreq, bool retrieve, uint32_t flags, Plan& pl) {
@@ -600,6 +650,10 @@ int copy_call(const kvs_geometry* g, const kvs_paged_cache* cache, const kvs_req
     Plan pl;
     int rc = validate_call(g, cache, reqs, nreq, pl);
     if (rc) return rc;
+    if (flags & KVS_F_VALIDATE) {
+        rc = check_overlaps(g, cache, reqs, nreq, retrieve);
+        if (rc) return rc;
+    }
     const int L = g->num_layers;
     const int lps = layers_per_step > 0 ? std::min(layers_per_step, L) : L;
     const int groups = (L + lps - 1) / lps;

@@ -84,6 +84,36 @@ def test_null_base_pointer_is_rejected():
     assert got == kvs.KVS_ERR_INVALID_ARG
 
 
+PLANES = [0x100000 + 4096 * p for p in range(4)]   # G: a plane is 8 blocks x 4 rows x 32 B = 1 KiB
+
+
+@pytest.mark.parametrize("fn,planes,reqs,alias", [
+    # two planes on the same memory: retrieve writes both
+    (kvs.kvs_retrieve, [PLANES[0], PLANES[0], PLANES[2], PLANES[3]], None, True),
+    # the same for a store only reads them
+    (kvs.kvs_store, [PLANES[0], PLANES[0], PLANES[2], PLANES[3]], None, False),
+    # a source chunk inside a plane that the retrieve writes
+    (kvs.kvs_retrieve, PLANES, "chunk_in_plane", True),
+    # store destinations overlapping each other (1 KiB chunks 512 B apart)
+    (kvs.kvs_store, PLANES, "chunks_overlap", True),
+    # ... which a retrieve only reads
+    (kvs.kvs_retrieve, PLANES, "chunks_overlap", False),
+], ids=["retrieve_planes", "store_planes", "retrieve_chunk_in_plane", "store_chunks", "retrieve_chunks"])
+def test_validate_reports_overlapping_memory(fn, planes, reqs, alias):
+    """With KVS_F_VALIDATE, memory a call writes may overlap neither itself nor what it
+    reads (checked on the host before any device work)."""
+    r = _req()
+    if reqs == "chunk_in_plane":
+        r.chunks[1].base = PLANES[2] + 256
+    elif reqs == "chunks_overlap":
+        r.chunks[1].base = r.chunks[0].base + 512
+    got, msg = _code(fn=fn, planes=planes, reqs=[r], flags=kvs.KVS_F_VALIDATE)
+    if alias:
+        assert got == kvs.KVS_ERR_ALIAS and "overlaps" in msg, msg
+    else:
+        assert got != kvs.KVS_ERR_ALIAS, msg       # passes the check; fails later without a GPU
+
+
 def test_call_too_large_is_rejected():
     # 2^31 pieces or more: 32768 layers, B = 1, 128 chunks of 256 tokens
     geom = (32768, 1, 8, 2, 1, 256)
