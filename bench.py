@@ -55,6 +55,8 @@ def parse_args(argv=None):
                     help="TempoKV control-plane model driven by the retrieval rate measured in this run")
     ap.add_argument("--sizes", action="store_true",
                     help="llama8b shape: retrieval rate against call size (1 to 128 chunks)")
+    ap.add_argument("--tier", action="store_true",
+                    help="llama8b: claims staged into the fast-tier ledger's pinned arena, retrieved from its slots")
     ap.add_argument("--duplex", action="store_true",
                     help="llama8b: retrieval (host->GPU) and store-back (GPU->host) at the same time")
     ap.add_argument("--side-priority", choices=["normal", "high"], default="high",
@@ -1108,6 +1110,96 @@ def run_sizes(args):
     return 0
 
 
+def run_tier(args):
+    """The 8B-shaped batch retrieved from the fast tier's own pinned arena: each request's
+    chunks are committed as one claim (its ordered manifest), staged into arena slots (a
+    host copy stands in for the SSD read), retrieved from the slots the ledger hands out,
+    and released.  The planes must equal those of a retrieval from the ordinary pinned
+    pool.  Reports the arena retrieval rate against the host link, the staging copy
+    rate, the ledger's cost per operation and the protected byte-time C."""
+    import ctypes
+    import numpy as np
+    import torch
+    from paper_2609_35065_gb300 import buffers, kvs, synth
+
+    torch.cuda.set_device(0)
+    kvs.lib()
+    stream = torch.cuda.Stream()
+    bw = kvs.kvs_query_bw(stream, 1 << 30)
+    host_peak = max(bw["h2d_copy_engine_gbs"], bw["zero_copy_read_gbs"])
+    w = workload("llama8b")
+    g = w.geom
+    buf = buffers.allocate(w)
+    chunk_bytes = g.chunk_tokens * token_bytes(g)
+    n_obj = sum(len(r.chunks) for r in buf.requests)
+    tier = kvs.Tier(n_obj + 32, n_obj + 8, chunk_bytes, arena=True)
+    keys = {r: [r * 1000 + j for j in range(len(q.chunks))] for r, q in enumerate(buf.requests)}
+    clock0 = time.perf_counter()
+
+    def now():
+        return time.perf_counter() - clock0
+
+    op_us = {"commit": [], "staged": [], "begin_retrieval": [], "end_retrieval": []}
+
+    def timed(name, fn, *a):
+        t = time.perf_counter()
+        out = fn(*a)
+        op_us[name].append((time.perf_counter() - t) * 1e6)
+        return out
+
+    stage_s = 0.0
+    for r, q in enumerate(buf.requests):
+        for k in timed("commit", tier.commit, r + 1, keys[r], now()):
+            dst = tier.slot_address(tier.object(k)["slot"])
+            t = time.perf_counter()
+            ctypes.memmove(dst, q.chunks[k % 1000].base.data_ptr(), chunk_bytes)   # the "SSD read"
+            stage_s += time.perf_counter() - t
+            timed("staged", tier.staged, k, now())
+    areqs = []
+    for r, q in enumerate(buf.requests):
+        slots = timed("begin_retrieval", tier.begin_retrieval, r + 1, now(), len(keys[r]))
+        areqs.append(kvs.RequestArg(q.block_table, [kvs.ChunkArg(tier.slot_address(sl), c.num_tokens)
+                                                    for sl, c in zip(slots, q.chunks)], q.first_token))
+    # bit-exact against a retrieval of the same batch from the ordinary pinned pool
+    kvs.kvs_retrieve(g, buf.plane_ptrs, w.num_blocks, buf.requests, stream, kvs.KVS_F_VALIDATE)
+    ref = buf.planes.clone()
+    buf.planes.fill_(int(np.array([synth.SENTINEL_BF16], dtype=np.uint16).view(np.int16)[0]))
+    torch.cuda.synchronize()
+    kvs.kvs_retrieve(g, buf.plane_ptrs, w.num_blocks, areqs, stream, kvs.KVS_F_VALIDATE)
+    torch.cuda.synchronize()
+    equal = bool(torch.equal(ref, buf.planes))
+    del ref
+    reps = max(3, min(args.steps, 20))
+    for _ in range(3):
+        kvs.kvs_retrieve(g, buf.plane_ptrs, w.num_blocks, areqs, stream, 0)
+    t0, t1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    t0.record(stream)
+    for _ in range(reps):
+        kvs.kvs_retrieve(g, buf.plane_ptrs, w.num_blocks, areqs, stream, 0)
+    t1.record(stream)
+    torch.cuda.synchronize()
+    ms = t0.elapsed_time(t1) / reps
+    for r in range(len(buf.requests)):
+        timed("end_retrieval", tier.end_retrieval, r + 1, now())
+    st = tier.stats(now())
+    gbs = buf.payload_bytes / (ms / 1e3) / 1e9
+    line = {"metric": METRIC + " (retrieval from the fast tier's arena, claims through the ledger)",
+            "unit": "GB/s", "value": round(gbs, 2),
+            "config": {"workload": describe(w), "tier": f"{n_obj + 32} slots of {chunk_bytes >> 20} MiB, "
+                       f"budget {n_obj + 8} objects, pinned arena", "claims": len(buf.requests),
+                       "timing": f"{reps} back-to-back retrievals while every claim is Transferring"},
+            "bit_exact_vs_pool": equal,
+            "frac_of_host_link": round(gbs / host_peak, 4),
+            "staging_copy_gbs": round(n_obj * chunk_bytes / stage_s / 1e9, 2),
+            "ledger_us_per_op": {k: round(statistics.median(v), 1) for k, v in op_us.items()},
+            "tier_stats": st,
+            "cost_C_gib_s_per_request": round(st["protected_object_seconds"] * chunk_bytes / 2 ** 30
+                                              / max(1, st["completed"]), 4)}
+    print(json.dumps(line), flush=True)
+    tier.close()
+    return 0 if equal else 1
+
+
 def main(argv=None):
     args = parse_args(argv)
     if args.tempokv:
@@ -1122,6 +1214,8 @@ def main(argv=None):
         return run_duplex(args)
     if args.sizes:
         return run_sizes(args)
+    if args.tier:
+        return run_tier(args)
     return run_ours(args)
 
 
