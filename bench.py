@@ -104,9 +104,16 @@ def measured_peaks() -> dict:
         return {}
 
 
-def kernel_hash() -> str:
-    with open(KERNEL_SRC, "rb") as f:
-        return hashlib.sha256(f.read()).hexdigest()[:16]
+def kernel_hash(src: str | None = None) -> str:
+    """Hash of the kernel source with comments and whitespace removed: it changes
+    with the code, not with its commentary."""
+    import re
+    if src is None:
+        with open(KERNEL_SRC) as f:
+            src = f.read()
+    src = re.sub(r"/\*.*?\*/", " ", src, flags=re.S)
+    src = re.sub(r"//[^\n]*", " ", src)
+    return hashlib.sha256(" ".join(src.split()).encode()).hexdigest()[:16]
 
 
 def recorded_traffic(kernel: str, config: str):

@@ -5,17 +5,20 @@
 // between a chunk buffer [L][2][n][H][D] and one paged block of one
 // (layer, K/V) plane [NB][B][H][D].  Two flavours:
 //
-//  * LDG: all threads of a 256-thread CTA move one 32 KiB piece with
-//    16-byte vector loads (non-coherent, no L1 allocation) issued ahead of
-//    16-byte streaming stores; one CTA per piece (or a capped grid-stride
-//    grid).  Works for device and mapped-host sources and destinations.
+//  * LDG: the threads of a CTA move one 32 KiB piece with 16-byte vector
+//    loads (non-coherent, no L1 allocation) issued ahead of 16-byte streaming
+//    stores.  Uncapped 16-byte work runs one 512-thread, 28-register CTA per
+//    piece (kvs_ldg_piece_kernel, four CTAs per SM); capped grids, narrower
+//    vectors and the validation compare run a 256-thread grid-stride kernel.
 //  * LINK: the LDG scheme double-buffered in registers (the next piece's loads
 //    are issued before the current piece is stored), for host-resident
 //    chunks whose loads/stores cross the long-latency host link.
-//  * TMA: one thread per CTA drives a ring of shared-memory stages with 1-D
-//    bulk async copies (cp.async.bulk global->shared completing on an
-//    mbarrier, then shared->global bulk stores); every wait is bounded by the
-//    global timer and reports KVS_ERR_TIMEOUT instead of hanging.
+//  * TMA: 1-D bulk async copies through shared memory (cp.async.bulk
+//    global->shared completing on an mbarrier, then a shared->global bulk
+//    store).  Uncapped work runs one 32-thread CTA per piece (six per SM);
+//    a capped grid runs one thread per CTA driving a ring of stages.  Every
+//    wait is bounded by the global timer and reports KVS_ERR_TIMEOUT instead
+//    of hanging.
 #include <algorithm>
 #include <cstdint>
 
