@@ -630,8 +630,10 @@ int read_error_word(DevState& st, cudaStream_t s) {
 }
 
 // layers_per_step > 0: layer-wise copy, one launch group per `layers_per_step`
-// layers, each followed by a record of layer_events[group] (if given) on the
-// caller's stream.
+// layers, each preceded by a wait on ready_events[group] and followed by a
+// record of layer_events[group] (either if given) on the caller's stream; with
+// KVS_F_LAYER_SIGNAL (host chunks, events, no ready events) one resident launch
+// signals every group instead.
 int copy_call(const kvs_geometry* g, const kvs_paged_cache* cache, const kvs_request* reqs,
               int32_t nreq, void* stream, uint32_t flags, bool retrieve,
               int32_t layers_per_step = 0, void* const* layer_events = nullptr,
