@@ -22,6 +22,7 @@ VARIANTS = {
     "tma": kvs.KVS_F_FORCE_TMA,
     "hbmcopy_tma": kvs.KVS_F_FORCE_HBMCOPY | kvs.KVS_F_FORCE_TMA,
     "few_ctas": kvs.KVS_F_MAX_CTAS(3),
+    "tma_few_ctas": kvs.KVS_F_FORCE_TMA | kvs.KVS_F_MAX_CTAS(3),      # the persistent TMA pipeline
 }
 
 
@@ -84,7 +85,7 @@ def test_tiny_retrieve_then_store_round_trip(variant):
         assert torch.equal(a, b)
 
 
-@pytest.mark.parametrize("variant", ["default", "hbmcopy", "tma"])
+@pytest.mark.parametrize("variant", ["default", "hbmcopy", "tma", "tma_few_ctas"])
 def test_tiny_device_resident_source(variant):
     w = synth.tiny()
     w.requests[0].residency = "device"
@@ -130,7 +131,7 @@ def test_random_small_geometries(seed):
                  kvs.KVS_F_MAX_CTAS(1 + seed % 7)]
     row = g.row_elems * g.elem_bytes
     if row % 16 == 0:
-        flags_all.append(kvs.KVS_F_FORCE_TMA)
+        flags_all += [kvs.KVS_F_FORCE_TMA, kvs.KVS_F_FORCE_TMA | kvs.KVS_F_MAX_CTAS(2 + seed % 5)]
     flags = flags_all[seed % len(flags_all)]
     buf = buffers.allocate(w, store=True, store_residency="host" if seed % 2 else "device")
     _retrieve(buf, flags)
@@ -140,15 +141,18 @@ def test_random_small_geometries(seed):
     gc.check_store(buf)
 
 
-@pytest.mark.parametrize("kernel", ["ldg", "tma"])
+@pytest.mark.parametrize("kernel", ["ldg", "tma", "ldg_capped", "tma_capped"])
 @pytest.mark.parametrize("geometry", [(2, 8, 256), (3, 4, 128)], ids=["64KiB_runs", "16KiB_runs"])
 def test_per_piece_kernels_full_and_partial_pieces(kernel, geometry):
-    """Uncapped HBM copies run one CTA per 32 KiB piece.  With H8 D256 a block's run is
-    64 KiB (two pieces); with H4 D128 it is 16 KiB (one short piece).  The 700-token
-    request ends in a 188-token chunk whose last block holds 12 tokens, so full pieces,
-    partial pieces and partial blocks all occur, in both directions."""
+    """Uncapped HBM copies run one CTA per 32 KiB piece; a CTA cap selects the grid-stride
+    LDG kernel or the persistent TMA pipeline.  With H8 D256 a block's run is 64 KiB (two
+    pieces); with H4 D128 it is 16 KiB (one short piece).  The 700-token request ends in a
+    188-token chunk whose last block holds 12 tokens, so full pieces, partial pieces and
+    partial blocks all occur, in both directions."""
     L, H, D = geometry
-    flags = kvs.KVS_F_FORCE_LDG if kernel == "ldg" else kvs.KVS_F_FORCE_TMA
+    flags = kvs.KVS_F_FORCE_LDG if kernel.startswith("ldg") else kvs.KVS_F_FORCE_TMA
+    if kernel.endswith("capped"):
+        flags |= kvs.KVS_F_MAX_CTAS(7)
     w = synth.custom(L, H, D, 16, 256, 300, [1024, 700, 512], [1024, 700, 512], seed=5, dist="normal",
                      residency="device")
     buf = buffers.allocate(w)
