@@ -87,14 +87,15 @@ def test_store_layers_matches_oracle(lps):
     gc.check_store(buf)
 
 
+@pytest.mark.parametrize("dest", ["host", "device"])
 @pytest.mark.parametrize("lps", [1, 2])
-def test_store_layers_waits_for_each_groups_ready_event(lps):
+def test_store_layers_waits_for_each_groups_ready_event(lps, dest):
     """A producer stream rewrites layer group k's planes after a delay, then records
     ready[k]; the store must copy the rewritten bytes of every group (a store that did
     not wait would copy the planes' earlier contents)."""
     w = synth.custom(4, 8, 128, 16, 256, 128, [1024, 700], [0, 0], seed=11, store_tokens=[768, 700])
     g = w.geom
-    buf = buffers.allocate(w, store=True, plane_init="random")
+    buf = buffers.allocate(w, store=True, store_residency=dest, plane_init="random")
     groups = -(-g.layers // lps)
     gen = torch.Generator(device="cuda").manual_seed(3)
     fresh = torch.randint(-32768, 32767, tuple(buf.planes.shape), dtype=torch.int16, device="cuda", generator=gen)

@@ -123,7 +123,7 @@ def _random_workload(seed):
     return w
 
 
-@pytest.mark.parametrize("seed", range(24))
+@pytest.mark.parametrize("seed", range(40))
 def test_random_small_geometries(seed):
     w = _random_workload(seed)
     g = w.geom
