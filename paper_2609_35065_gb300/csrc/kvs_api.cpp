@@ -933,9 +933,9 @@ int query_bw(DevState& st, kvs_bw_report* out, cudaStream_t s, int64_t probe_byt
     st.hostlink_ctas = rep.hostlink_ctas;
     st.store_ctas = rep.store_ctas;
     // The probe's buffer is small.  On GB300 the copy engine's rate from pinned
-    // host memory falls on buffers of tens of GiB (to 100-180 GB/s on a 40 GiB
-    // fast tier, where SM loads keep the link's rate), so the copy-engine
-    // variant is taken only when it wins the probe clearly.
+    // host memory is erratic on buffers of tens of GiB (13-210 GB/s on 40 GiB,
+    // by box and allocation), where SM loads keep the link's rate, so the
+    // copy-engine variant is taken only when it wins the probe clearly.
     constexpr double kHbmcopyMargin = 1.05;
     st.retrieve_host = rep.retrieve_gbs[1] > kHbmcopyMargin * rep.retrieve_gbs[0] ? KVS_VARIANT_HBMCOPY
                                                                                  : KVS_VARIANT_HOSTLINK;
