@@ -61,6 +61,8 @@ def parse_args(argv=None):
                     help="llama8b: retrieval (host->GPU) and store-back (GPU->host) at the same time")
     ap.add_argument("--side-priority", choices=["normal", "high"], default="high",
                     help="priority of the retrieval stream in --overlap runs")
+    ap.add_argument("--no-extras", action="store_true",
+                    help="default line without its extra legs (no-alloc, store to host, sweep50, overlap)")
     return ap.parse_args(argv)
 
 
@@ -117,16 +119,25 @@ def kernel_hash(src: str | None = None) -> str:
 
 
 def recorded_traffic(kernel: str, config: str):
-    """Per-launch DRAM bytes from an ncu capture of the current kernel source, else None."""
+    """(per-launch DRAM bytes, provenance) from an ncu capture recorded for the current
+    kernel source, else (None, why).  The bytes are a stored record, not measured in
+    this run: the provenance says which capture and source hash they come from."""
     try:
         with open(TRAFFIC_FILE) as f:
             rec = json.load(f)
     except (OSError, ValueError):
-        return None
+        return None, {"kind": "none", "why": "no recorded capture"}
     ent = rec.get(f"{config}/{kernel}")
-    if not ent or ent.get("kernel_sha") != kernel_hash():
-        return None
-    return ent.get("dram_bytes_per_launch")
+    sha = kernel_hash()
+    if not ent:
+        return None, {"kind": "none", "why": f"no recorded capture of {kernel} on {config}"}
+    if ent.get("kernel_sha") != sha:
+        return None, {"kind": "stale", "why": "kernel source changed since the capture",
+                      "capture_kernel_sha": ent.get("kernel_sha"), "kernel_sha": sha}
+    prov = {"kind": "recorded", "kernel_sha": sha, "capture": ent.get("capture", "profiles/traffic.json")}
+    if "scaled_from" in ent:
+        prov["scaled_from"] = ent["scaled_from"]
+    return ent.get("dram_bytes_per_launch"), prov
 
 
 class ClockSampler:
@@ -383,8 +394,6 @@ def run_ours(args):
     wall1 = time.time()
     barrier()
     launches = kvs.kvs_stat_launches() - launches0
-    time.sleep(0.1)
-    sampler.stop()
     total_ms = max_over_ranks(t_start.elapsed_time(t_end), dist, "cuda")
     per_call_ms = [a.elapsed_time(b) for a, b in ev]
     call_ms = statistics.mean(per_call_ms)
@@ -459,17 +468,24 @@ def run_ours(args):
         dev_ms = [a.elapsed_time(b) for a, b in dev_ev]
         dms = statistics.mean(dev_ms)
         peaks = measured_peaks()
-        hpk = peaks.get("hbm_gbs", HBM_FALLBACK_GBS)
+        # the roofline is the faster of the driver's copy measurement and our own
+        # flat copy kernel in this run (both count read + write bytes)
+        drv_pk = peaks.get("hbm_gbs", HBM_FALLBACK_GBS)
+        hpk = max(drv_pk, bw["hbm_copy_gbs"])
+        hpk_src = ("in-run flat copy kernel (kvs_query_bw hbm_copy_gbs, read+write bytes)" if hpk > drv_pk else
+                   "MEASURED_PEAKS.json hbm_gbs (copy, read+write bytes)" if peaks else "fallback")
         ach = 2 * payload / (dms / 1e3) / 1e9
         tma = args.kernel == "tma" or (args.kernel == "auto" and choice["chosen_kernel_device"] == 2)
         if args.max_ctas:
             kname = "kvs_tma_kernel" if tma else "kvs_ldg_kernel"
         else:
             kname = "kvs_tma_piece_kernel" if tma else "kvs_ldg_piece_kernel"
-        hbm = {"bound": "hbm", "achieved": round(ach, 1), "peak": hpk, "unit": "GB/s",
-               "frac": round(ach / hpk, 4), "traffic": recorded_traffic(kname, "llama8b_device"),
+        tr, tr_src = recorded_traffic(kname, "llama8b_device")
+        hbm = {"bound": "hbm", "achieved": round(ach, 1), "peak": round(hpk, 1), "unit": "GB/s",
+               "frac": round(ach / hpk, 4), "traffic": tr, "traffic_source": tr_src,
                "kernel": kname, "payload_gbs": round(payload / (dms / 1e3) / 1e9, 1),
-               "peak_source": "MEASURED_PEAKS.json hbm_gbs (copy, read+write bytes)" if peaks else "fallback",
+               "peak_source": hpk_src, "measured_peaks_hbm_gbs": drv_pk,
+               "frac_of_measured_peaks": round(ach / drv_pk, 4),
                "bytes_counted": "2 x payload (read + write)"}
 
         # store-back (gather) of the same blocks into the HBM-resident chunks
@@ -487,8 +503,11 @@ def run_ours(args):
         torch.cuda.synchronize()
         sms = statistics.mean(a.elapsed_time(b) for a, b in st_ev)
         sach = 2 * payload / (sms / 1e3) / 1e9
-        hbm_store = {"bound": "hbm", "achieved": round(sach, 1), "peak": hpk, "unit": "GB/s",
-                     "frac": round(sach / hpk, 4), "traffic": recorded_traffic(kname, "llama8b_device_store"),
+        tr, tr_src = recorded_traffic(kname, "llama8b_device_store")
+        hbm_store = {"bound": "hbm", "achieved": round(sach, 1), "peak": round(hpk, 1), "unit": "GB/s",
+                     "frac": round(sach / hpk, 4), "traffic": tr, "traffic_source": tr_src,
+                     "peak_source": hpk_src, "measured_peaks_hbm_gbs": drv_pk,
+                     "frac_of_measured_peaks": round(sach / drv_pk, 4),
                      "kernel": kname,
                      "payload_gbs": round(payload / (sms / 1e3) / 1e9, 1),
                      "bytes_counted": "2 x payload (read + write)"}
@@ -540,14 +559,19 @@ def run_ours(args):
                                  "unit": "GB/s", "cores": 1,
                                  "sample": f"planes 0-{len(sub) - 1} of {2 * g.layers} (same bytes per plane)"}}
 
+    if rank == 0 and world == 1 and w.name == "llama8b" and not args.no_extras:
+        extras.update(default_line_legs(args, buf, bw, stream, sampler, flags))
+    time.sleep(0.1)
+    sampler.stop()
     clocks = sampler.summary(wall0, wall1)
     mv = moved_bytes(w)
     hbm_peak = measured_peaks().get("hbm_gbs", HBM_FALLBACK_GBS)
     if mv["device"] == 0:
         achieved = mv["host"] / (call_ms / 1e3) / 1e9
+        tr, tr_src = recorded_traffic(kernel_name, w.name)
         roofline = {"bound": "host_link", "achieved": round(achieved, 2), "peak": round(host_peak, 2),
                     "unit": "GB/s", "frac": round(achieved / host_peak, 4),
-                    "traffic": recorded_traffic(kernel_name, w.name), "kernel": kernel_name,
+                    "traffic": tr, "traffic_source": tr_src, "kernel": kernel_name,
                     "peak_source": "measured in this run: max(copy-engine pinned H2D, zero-copy read kernel)",
                     "bytes_counted": f"bytes moved over the host link per step ({mv['host']})"}
     else:
@@ -590,24 +614,21 @@ def run_ours(args):
     return 0
 
 
-def run_overlap(args):
-    """Retrieval of the 70B-shaped batch on a side stream while the main stream runs a
-    bf16 8192 x 8192 GEMM loop; the pinned fast-tier buffer holds buffer_frac of the
-    batch and is refilled between passes (untimed)."""
+def overlap_measure(w, bw, side, variants, sampler=None):
+    """Retrieval of workload ``w`` on the ``side`` stream while the current stream runs a
+    bf16 8192 x 8192 GEMM loop, for each (name, flags) of ``variants``, alone and beside the
+    GEMM.  The pinned fast-tier buffer holds ``w.notes['buffer_frac']`` of the batch and is
+    refilled between passes (untimed).  Returns {name: {"alone": ..., "with_gemm": ...}},
+    with the clocks of each GEMM window when ``sampler`` is given."""
     import torch
-    from paper_2609_35065_gb300 import buffers, kvs, synth
+    from paper_2609_35065_gb300 import kvs, synth
 
-    torch.cuda.set_device(0)
-    kvs.lib()
-    w = workload(args.config)
     g = w.geom
     frac = w.notes.get("buffer_frac", 1.0)
     passes = max(1, int(round(1 / frac)))
     per_pass = len(w.requests) // passes
     per_tok = 2 * g.layers * g.row_elems
     main = torch.cuda.current_stream()
-    side = torch.cuda.Stream(priority=-1 if args.side_priority == "high" else 0)
-    bw = kvs.kvs_query_bw(side, 1 << 30)
     host_peak = max(bw["h2d_copy_engine_gbs"], bw["zero_copy_read_gbs"])
     n = w.num_blocks * g.block_size * g.row_elems
     planes = torch.full((2 * g.layers, n), synth.SENTINEL_BF16, dtype=torch.int16, device="cuda")
@@ -634,6 +655,7 @@ def run_overlap(args):
     a = torch.randn(8192, 8192, dtype=torch.bfloat16, device="cuda")
     b = torch.randn(8192, 8192, dtype=torch.bfloat16, device="cuda")
     c = torch.empty(8192, 8192, dtype=torch.bfloat16, device="cuda")
+
     def ev():
         return torch.cuda.Event(enable_timing=True)
 
@@ -688,7 +710,8 @@ def run_overlap(args):
             kvs.kvs_retrieve(g, ptrs, w.num_blocks, reqs, side, flags)
 
     def retrieval(flags, with_gemm):
-        total_ms, gemm_n, gemm_during, gemm_alone = 0.0, 0, [], []
+        total_ms, gemm_during, gemm_alone = 0.0, [], []
+        wall = [time.time(), None]
         for k in range(passes):
             if k:
                 pinned.copy_(refill_src)                 # refill between passes (untimed)
@@ -711,15 +734,140 @@ def run_overlap(args):
             gemm_during.append(rate_within(g0, gev, r_ms))
             a0, aev, _ = gemm_window(iters)
             gemm_alone.append(rate_within(a0, aev, r_ms))
+        wall[1] = time.time()
         gbs = passes * tokens_pass * per_tok * 2 / (total_ms / 1e3) / 1e9
         out = {"retrieval_gbs": round(gbs, 2), "frac_of_host_link": round(gbs / host_peak, 4)}
         if with_gemm:
             during, alone = statistics.mean(gemm_during), statistics.mean(gemm_alone)
             out.update({"gemm_tflops_during": round(during, 1), "gemm_tflops_alone_same_window": round(alone, 1),
                         "gemm_kept": round(during / alone, 4)})
+            if sampler is not None:
+                out["clocks"] = sampler.summary(*wall)
         return out
 
     results = {}
+    for name, fl in variants:
+        results[name] = {"alone": retrieval(fl, False), "with_gemm": retrieval(fl, True)}
+    info = {"buffer_frac": frac, "passes": passes, "host_link_peak_gbs": round(host_peak, 2),
+            "gemm": "bf16 8192x8192x8192 torch.matmul loop on the main stream",
+            "gemm_tflops_short_burst": round(2 * 8192 ** 3 / (gemm_ms / 1e3) / 1e12, 1)}
+    del planes, pinned, refill_src, a, b, c
+    torch.cuda.empty_cache()
+    return results, info
+
+
+def default_line_legs(args, buf, bw, stream, sampler, flags):
+    """Extra legs of the default line, each a short window with its own clock record:
+
+    * ``noalloc``: the same 4 GiB batch through kvs_retrieve_noalloc (allocation-free
+      entry point), next to kvs_retrieve's rate;
+    * ``store_host``: the batch stored back from the paged cache into its pinned host
+      chunks (the store-back direction over the host link);
+    * ``sweep50``: the mixed-residency sweep at 50% prefix hit (32 requests x 4096
+      matched tokens, half in HBM staging, half in pinned host memory) into the same
+      20,000-block cache, with each source class alone;
+    * ``overlap``: the 70B-shaped batch (pinned buffer of 25%, 4 passes, refilled
+      between passes) retrieved on a high-priority side stream beside a bf16 8192^3
+      GEMM loop, at the default CTA cap.
+    """
+    import torch
+    from paper_2609_35065_gb300 import buffers, kvs, synth
+
+    w = buf.workload
+    g = w.geom
+    payload = buf.payload_bytes
+    host_peak = max(bw["h2d_copy_engine_gbs"], bw["zero_copy_read_gbs"])
+    d2h_peak = max(bw["d2h_copy_engine_gbs"], bw["zero_copy_write_gbs"])
+    hbm_peak = max(measured_peaks().get("hbm_gbs", HBM_FALLBACK_GBS), bw["hbm_copy_gbs"])
+    n = max(5, min(args.steps, 20))
+    legs = {}
+
+    def timed(fn):
+        """Mean and best seconds of n back-to-back calls of fn (CUDA events on `stream`),
+        and the wall-clock window they ran in."""
+        fn()
+        torch.cuda.synchronize()
+        evs = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)) for _ in range(n)]
+        t0 = time.time()
+        for a, b in evs:
+            a.record(stream)
+            fn()
+            b.record(stream)
+        torch.cuda.synchronize()
+        t1 = time.time()
+        ms = [a.elapsed_time(b) for a, b in evs]
+        return statistics.mean(ms) / 1e3, min(ms) / 1e3, (t0, t1)
+
+    # the allocation-free entry point on the same batch (host chunks: the link kernel on
+    # kvs_retrieve's cap), and kvs_retrieve again over the same window length
+    kvs.kvs_retrieve_noalloc(g, buf.plane_ptrs, w.num_blocks, buf.requests, stream, kvs.KVS_F_VALIDATE)
+    sec, best, win = timed(lambda: kvs.kvs_retrieve_noalloc(g, buf.plane_ptrs, w.num_blocks, buf.requests,
+                                                            stream, flags & 0xFFFF0000))
+    ref, _, _ = timed(lambda: kvs.kvs_retrieve(g, buf.plane_ptrs, w.num_blocks, buf.requests, stream, flags))
+    legs["noalloc"] = {"gbs": round(payload / sec / 1e9, 2), "best_gbs": round(payload / best / 1e9, 2),
+                       "frac_of_host_link": round(payload / sec / 1e9 / host_peak, 4),
+                       "kvs_retrieve_gbs_same_window": round(payload / ref / 1e9, 2), "calls": n,
+                       "kernel": "kvs_link_kernel (host chunks, kvs_retrieve's CTA cap)",
+                       "clocks": sampler.summary(*win)}
+
+    # store-back of the same blocks into the pinned host chunks
+    kvs.kvs_store(g, buf.plane_ptrs, w.num_blocks, buf.requests, stream, kvs.KVS_F_VALIDATE)
+    sec, best, win = timed(lambda: kvs.kvs_store(g, buf.plane_ptrs, w.num_blocks, buf.requests, stream, 0))
+    choice = kvs.kvs_get_choice()
+    legs["store_host"] = {"gbs": round(payload / sec / 1e9, 2), "best_gbs": round(payload / best / 1e9, 2),
+                          "frac_of_d2h_link": round(payload / sec / 1e9 / d2h_peak, 4),
+                          "d2h_link_peak_gbs": round(d2h_peak, 2), "bytes": payload, "calls": n,
+                          "variant": {1: "hostlink", 2: "hbmcopy"}[choice["chosen_store_host"]],
+                          "ctas": choice["store_ctas"], "clocks": sampler.summary(*win)}
+
+    # mixed residency at 50% prefix hit, into the same cache (same geometry and block pool)
+    ws = synth.sweep(0.5)
+    sb = buffers.allocate(ws, with_planes=False)
+    mv = moved_bytes(ws)
+    spay = mv["host"] + mv["device"]
+
+    def sweep_call(reqs, f=0):
+        kvs.kvs_retrieve(g, buf.plane_ptrs, ws.num_blocks, reqs, stream, f)
+
+    sweep_call(sb.requests, kvs.KVS_F_VALIDATE)
+    sec, best, win = timed(lambda: sweep_call(sb.requests))
+    ideal = max(mv["host"] / (host_peak * 1e9), 2 * mv["device"] / (hbm_peak * 1e9))
+    leg = {"gbs": round(spay / sec / 1e9, 2), "tokens_per_s": round(ws.matched_tokens / sec, 1),
+           "frac_of_roofline": round(ideal / sec, 4), "bytes": spay, "calls": n,
+           "roofline": "max(host bytes / host-link peak, 2 x device bytes / HBM peak)",
+           "clocks": sampler.summary(*win)}
+    for cls in ("host", "device"):
+        sub = [ra for ra, r in zip(sb.requests, ws.requests) if r.residency == cls]
+        csec, _, _ = timed(lambda: sweep_call(sub))
+        cb = mv[cls]
+        leg[f"class_{cls}"] = {"gbs": round(cb / csec / 1e9, 2), "bytes": cb,
+                               "frac": round(cb / csec / 1e9 / host_peak, 4) if cls == "host"
+                               else round(2 * cb / csec / 1e9 / hbm_peak, 4)}
+    legs["sweep50"] = leg
+    del sb
+    torch.cuda.empty_cache()
+
+    # retrieval beside a bf16 GEMM loop (70B shape, 25% buffer), default cap
+    side = torch.cuda.Stream(priority=-1)
+    w70 = synth.llama70b(buffer_frac=0.25)
+    results, info = overlap_measure(w70, bw, side, [("default", 0)], sampler)
+    legs["overlap"] = {"workload": describe(w70), **info, "hostlink_ctas": kvs.kvs_get_choice()["hostlink_ctas"],
+                       "side_stream": "high priority", **results}
+    return legs
+
+
+def run_overlap(args):
+    """Retrieval of the 70B-shaped batch on a side stream while the main stream runs a
+    bf16 8192 x 8192 GEMM loop; the pinned fast-tier buffer holds buffer_frac of the
+    batch and is refilled between passes (untimed)."""
+    import torch
+    from paper_2609_35065_gb300 import kvs
+
+    torch.cuda.set_device(0)
+    kvs.lib()
+    w = workload(args.config)
+    side = torch.cuda.Stream(priority=-1 if args.side_priority == "high" else 0)
+    bw = kvs.kvs_query_bw(side, 1 << 30)
     variants = [("default", 0), ("hostlink_full", kvs.KVS_F_FORCE_HOSTLINK | kvs.KVS_F_MAX_CTAS(bw["num_sms"] * 3)),
                 ("hostlink_8ctas", kvs.KVS_F_FORCE_HOSTLINK | kvs.KVS_F_MAX_CTAS(8)),
                 ("hostlink_12ctas", kvs.KVS_F_FORCE_HOSTLINK | kvs.KVS_F_MAX_CTAS(12)),
@@ -727,13 +875,11 @@ def run_overlap(args):
                 ("hbmcopy", kvs.KVS_F_FORCE_HBMCOPY),
                 ("layer_launches", kvs.KVS_F_LAYER_LAUNCHES),
                 ("layer_launches_96ctas", kvs.KVS_F_LAYER_LAUNCHES | kvs.KVS_F_MAX_CTAS(96))]
-    for name, fl in variants:
-        results[name] = {"alone": retrieval(fl, False), "with_gemm": retrieval(fl, True)}
+    sampler = ClockSampler(torch.cuda.current_device())
+    results, info = overlap_measure(w, bw, side, variants, sampler)
+    sampler.stop()
     line = {"metric": METRIC + " (overlap with a bf16 GEMM loop)", "unit": "GB/s",
-            "config": {"workload": describe(w), "buffer_frac": frac, "passes": passes,
-                       "gemm": "bf16 8192x8192x8192 torch.matmul loop on the main stream"},
-            "gemm_tflops_short_burst": round(2 * 8192 ** 3 / (gemm_ms / 1e3) / 1e12, 1),
-            "host_link_peak_gbs": round(host_peak, 2),
+            "config": {"workload": describe(w), **info},
             "side_stream_priority": args.side_priority, "hostlink_ctas_default": bw["hostlink_ctas"],
             "variants": results}
     print(json.dumps(line), flush=True)

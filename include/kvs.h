@@ -304,14 +304,20 @@ int64_t kvs_stat_launches(void);
  *    KVS_ERR_UNSUPPORTED with a message saying so;
  *  - the first call on a device looks up the device address of that array
  *    (once per device, with that device current); make that first call
- *    before any stream capture;
+ *    before any stream capture.  kvs_shutdown() forgets the address, so
+ *    after a cudaDeviceReset call kvs_shutdown() before the next call;
  *  - every call shares the one array and overwrites it: calls whose work can
  *    overlap on the GPU (different streams, or other host threads) race and
- *    must be ordered by the caller; the error word is cleared at the start of
- *    each call;
- *  - host chunks are always read directly over the host link and every chunk
- *    is moved by the vector-load kernel (KVS_F_FORCE_HBMCOPY, KVS_F_FORCE_TMA
- *    and KVS_F_NO_DEDUP are refused with KVS_ERR_UNSUPPORTED);
+ *    must be ordered by the caller; calls in order on one stream are safe;
+ *    the error word is cleared at the start of each call;
+ *  - every chunk pointer is checked as kvs_retrieve's KVS_F_VALIDATE checks
+ *    it (mapped page-locked host memory, or device memory), on every call;
+ *  - host chunks are always read directly over the host link, by the same
+ *    double-buffered kernel and CTA cap as kvs_retrieve (KVS_F_MAX_CTAS
+ *    overrides the cap); device chunks take the vector-load kernel; the two
+ *    classes run one after the other on cuda_stream (KVS_F_FORCE_HBMCOPY,
+ *    KVS_F_FORCE_TMA and KVS_F_NO_DEDUP are refused with
+ *    KVS_ERR_UNSUPPORTED);
  *  - device-side errors are only reported with KVS_F_VALIDATE.
  */
 #define KVS_NOALLOC_SCRATCH_BYTES (1u << 20)

@@ -954,6 +954,23 @@ int query_bw(DevState& st, kvs_bw_report* out, cudaStream_t s, int64_t probe_byt
 
 void set_last_error(const char* msg) { t_error = msg; }
 
+int hostlink_grid(bool retrieve) {
+    std::lock_guard<std::mutex> lk(g_mu);
+    int dev = 0;
+    if (cudaGetDevice(&dev) != cudaSuccess) {
+        cudaGetLastError();
+        return 0;
+    }
+    if (dev < (int)g_dev.size() && g_dev[dev].ready)
+        return retrieve ? g_dev[dev].hostlink_ctas : g_dev[dev].store_ctas;
+    int sms = 0;
+    if (cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess) {
+        cudaGetLastError();
+        return 0;
+    }
+    return std::max(8, sms / 3);          // the built-in default of get_state
+}
+
 }  // namespace kvs
 
 using namespace kvs;
@@ -1079,6 +1096,7 @@ int kvs_shutdown(void) {
         st = DevState{};
     }
     g_dev.clear();
+    noalloc_forget_devices();
     cudaSetDevice(prev);
     return KVS_OK;
 }

@@ -77,6 +77,13 @@ cudaError_t launch_link_signal(const Job& job, const Signal& sig, int grid, cuda
 cudaError_t launch_stall(int32_t* err, uint64_t limit_ns, cudaStream_t s);
 // Sets the calling thread's message returned by kvs_last_error() (kvs_api.cpp).
 void set_last_error(const char* msg);
+// CTA cap kvs_retrieve / kvs_store give host-link kernels on the current device
+// (the measured one after kvs_query_bw, else the built-in default); allocates
+// nothing (kvs_api.cpp).
+int hostlink_grid(bool retrieve);
+// Forgets the per-device address of the allocation-free entry point's static
+// scratch (kvs_noalloc.cu); kvs_shutdown calls it.
+void noalloc_forget_devices();
 // CTAs per SM the flavour runs with (occupancy); used to size persistent grids.
 int ldg_ctas_per_sm();
 int link_ctas_per_sm();

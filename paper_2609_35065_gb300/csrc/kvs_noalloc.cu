@@ -11,9 +11,12 @@
 // the library image, which every GPU that loads the library holds until the
 // process exits.  Host-side planning uses static storage as well.
 //
-// The same LDG copy kernel as kvs_retrieve moves the bytes; only where its
-// scratch lives differs.  Host chunks are read directly over the host link
-// (no copy-engine staging ring, which would need an allocation).
+// The same copy kernels as kvs_retrieve move the bytes; only where their
+// scratch lives differs.  Host chunks are read directly over the host link by
+// the double-buffered link kernel on kvs_retrieve's CTA cap (no copy-engine
+// staging ring, which would need an allocation); device chunks take the vector
+// LDG kernel.  The two classes run one after the other on the caller's stream
+// (kvs_retrieve runs them side by side on two streams).
 #include <algorithm>
 #include <cstdarg>
 #include <cstdio>
@@ -37,8 +40,11 @@ void* g_dev_addr[kMaxDevices];                  // device address of g_scratch, 
 bool g_dev_ready[kMaxDevices];
 
 // Host staging, copied into g_scratch by one cudaMemcpyAsync per call.  The
-// copy reads pageable memory, so it is staged before cudaMemcpyAsync returns
-// and the array may be refilled by the next call at once.
+// source is pageable memory: the CUDA runtime documents that an asynchronous
+// copy from pageable host memory to device memory returns only once the source
+// has been copied to a staging buffer, so the next call may refill g_stage at
+// once while the previous upload is still queued on the stream.
+
 unsigned char g_stage[KVS_NOALLOC_SCRATCH_BYTES];
 uint64_t g_keys[kMaxBlockRefs];                  // (physical block << 32) | block-ref index
 int32_t  g_ref_req[kMaxBlockRefs];               // request of each block-ref
@@ -81,6 +87,28 @@ int scratch_address(void** out) {
     return KVS_OK;
 }
 
+// Device-visible address of a chunk, checked against its residency the way
+// kvs_retrieve checks it: a host chunk must be page-locked host memory mapped
+// into the GPU (its device pointer is used), a device chunk device memory.
+// Anything else is refused before any work is enqueued.
+int chunk_address(const kvs_chunk& c, int32_t r, int32_t j, uint64_t* out) {
+    cudaPointerAttributes at{};
+    if (cudaPointerGetAttributes(&at, c.base) != cudaSuccess) {
+        cudaGetLastError();
+        return na_fail(KVS_ERR_INVALID_ARG, "request %d chunk %d: unknown pointer", r, j);
+    }
+    if (c.residency == KVS_SRC_DEVICE) {
+        if (!(at.type == cudaMemoryTypeDevice || at.type == cudaMemoryTypeManaged))
+            return na_fail(KVS_ERR_INVALID_ARG, "request %d chunk %d: not device memory", r, j);
+        *out = (uint64_t)c.base;
+    } else {
+        if (at.type != cudaMemoryTypeHost || !at.devicePointer)
+            return na_fail(KVS_ERR_INVALID_ARG, "request %d chunk %d: not mapped page-locked host memory", r, j);
+        *out = (uint64_t)at.devicePointer;
+    }
+    return KVS_OK;
+}
+
 int retrieve_noalloc(const kvs_geometry* g, const kvs_paged_cache* cache, const kvs_request* reqs,
                      int32_t nreq, cudaStream_t s, uint32_t flags) {
     const uint32_t allowed = KVS_F_VALIDATE | KVS_F_FORCE_HOSTLINK | KVS_F_FORCE_LDG | 0xFFFF0000u;
@@ -110,7 +138,7 @@ int retrieve_noalloc(const kvs_geometry* g, const kvs_paged_cache* cache, const 
         if (!cache->kv_planes[p]) return na_fail(KVS_ERR_INVALID_ARG, "plane %d is NULL", p);
         addr_or |= (uint64_t)cache->kv_planes[p];
     }
-    uint64_t nent = 0;
+    uint64_t nent = 0, ndev = 0;
     for (int32_t r = 0; r < nreq; ++r) {
         const kvs_request& q = reqs[r];
         if (q.first_token < 0 || q.first_token % C)
@@ -132,7 +160,7 @@ int retrieve_noalloc(const kvs_geometry* g, const kvs_paged_cache* cache, const 
             if (j + 1 < q.num_chunks && c.num_tokens != C)
                 return na_fail(KVS_ERR_INVALID_ARG, "request %d chunk %d: only the last chunk may be partial", r, j);
             sum += c.num_tokens;
-            addr_or |= (uint64_t)c.base;
+            if (c.residency == KVS_SRC_DEVICE) ++ndev;
         }
         if (sum != q.num_tokens)
             return na_fail(KVS_ERR_INVALID_ARG, "request %d: chunks hold %lld tokens, num_tokens is %lld",
@@ -171,13 +199,11 @@ int retrieve_noalloc(const kvs_geometry* g, const kvs_paged_cache* cache, const 
     if (nrefs * P * ppr >= (1ull << 31))
         return na_fail(KVS_ERR_INVALID_ARG, "call too large: split it (more than 2^31 pieces)");
 
-    void* dscratch = nullptr;
-    int rc = scratch_address(&dscratch);
-    if (rc) return rc;
-
-    // Pack the tables.  Block refs: one per (entry, block of its chunk); a ref
-    // of a physical block already written by an earlier request is dropped
-    // (the ref covering most tokens is kept, the lowest request on ties).
+    // Pack the tables: device-resident entries first, then host-resident ones,
+    // so that each class is one contiguous range of entries (one launch each).
+    // Block refs: one per (entry, block of its chunk); a ref of a physical
+    // block also named by another request is dropped unless it covers the
+    // most tokens of that block (the lowest request on ties).
     unsigned char* st = g_stage;
     memset(st, 0, off_bc);
     uint64_t* planes = (uint64_t*)(st + off_pl);
@@ -185,13 +211,18 @@ int retrieve_noalloc(const kvs_geometry* g, const kvs_paged_cache* cache, const 
     int32_t* blocks = (int32_t*)(st + off_bl);
     int32_t* demoted = (int32_t*)(st + off_bc);
     for (int p = 0; p < P; ++p) planes[p] = (uint64_t)cache->kv_planes[p];
-    uint32_t e = 0, nk = 0;
+    uint32_t e_dev = 0, e_host = (uint32_t)ndev, nk = 0;
     for (int32_t r = 0; r < nreq; ++r) {
         const kvs_request& q = reqs[r];
         int64_t s0 = q.first_token;
-        for (int32_t j = 0; j < q.num_chunks; ++j, ++e) {
+        for (int32_t j = 0; j < q.num_chunks; ++j) {
             const kvs_chunk& c = q.chunks[j];
-            entries[e].chunk = (uint64_t)c.base;
+            const uint32_t e = (c.residency == KVS_SRC_DEVICE) ? e_dev++ : e_host++;
+            uint64_t addr = 0;
+            int rc = chunk_address(c, r, j, &addr);
+            if (rc) return rc;
+            addr_or |= addr;
+            entries[e].chunk = addr;
             entries[e].n_tok = c.num_tokens;
             entries[e].pad = 0;
             for (uint32_t i = 0; i < bpc; ++i) {
@@ -209,6 +240,10 @@ int retrieve_noalloc(const kvs_geometry* g, const kvs_paged_cache* cache, const 
     }
     if (validate)
         for (uint64_t k = 0; k < nrefs; ++k) demoted[k] = -1;
+    // Sorted by (block, ref), the refs of one block are adjacent; within a
+    // block, refs of one request are adjacent too only if the request names
+    // the block twice, which is refused (checked against every earlier ref of
+    // the block by request).
     std::sort(g_keys, g_keys + nk);                         // in place: no allocation
     bool any_demoted = false;
     for (uint32_t a = 0; a < nk;) {
@@ -218,10 +253,15 @@ int retrieve_noalloc(const kvs_geometry* g, const kvs_paged_cache* cache, const 
         if (b - a > 1) {
             uint32_t keep = (uint32_t)g_keys[a];
             for (uint32_t k = a + 1; k < b; ++k) {
-                const uint32_t ref = (uint32_t)g_keys[k], prev = (uint32_t)g_keys[k - 1];
-                if (g_ref_req[ref] == g_ref_req[prev])
-                    return na_fail(KVS_ERR_ALIAS, "request %d names physical block %u twice", g_ref_req[ref], blk);
-                if (g_ref_ntok[ref] > g_ref_ntok[keep]) keep = ref;
+                const uint32_t ref = (uint32_t)g_keys[k];
+                for (uint32_t m = a; m < k; ++m)
+                    if (g_ref_req[(uint32_t)g_keys[m]] == g_ref_req[ref])
+                        return na_fail(KVS_ERR_ALIAS, "request %d names physical block %u twice",
+                                       g_ref_req[ref], blk);
+                const uint32_t kr = keep;
+                if (g_ref_ntok[ref] > g_ref_ntok[kr] ||
+                    (g_ref_ntok[ref] == g_ref_ntok[kr] && g_ref_req[ref] < g_ref_req[kr]))
+                    keep = ref;
             }
             for (uint32_t k = a; k < b; ++k) {
                 const uint32_t ref = (uint32_t)g_keys[k];
@@ -234,6 +274,9 @@ int retrieve_noalloc(const kvs_geometry* g, const kvs_paged_cache* cache, const 
         a = b;
     }
 
+    void* dscratch = nullptr;
+    int rc = scratch_address(&dscratch);
+    if (rc) return rc;
     unsigned char* d = (unsigned char*)dscratch;
     const size_t upload = validate && any_demoted ? need : off_bc;
     NA_CUDA(cudaMemsetAsync(d, 0, sizeof(int32_t), s));             // error word starts at zero
@@ -248,22 +291,42 @@ int retrieve_noalloc(const kvs_geometry* g, const kvs_paged_cache* cache, const 
     j.err = (int32_t*)d;
     j.row_bytes = R;
     j.num_blocks = cache->num_blocks;
-    j.num_entries = e;
-    j.entry_base = 0;
     j.num_planes = (uint32_t)P;
     j.plane_begin = 0;
     j.blocks_per_chunk = bpc;
     j.piece_bytes = kPieceBytes;
     j.block_size = (uint32_t)B;
     j.pieces_per_run = (uint32_t)ppr;
-    j.num_pieces = (uint64_t)e * P * bpc * ppr;
     j.mode = MODE_RETRIEVE;
-    const int grid = (int)KVS_F_GET_MAX_CTAS(flags);
-    NA_CUDA(launch_ldg(j, vec, grid, s));
+    const int cap = (int)KVS_F_GET_MAX_CTAS(flags);
+    // host-resident entries: the link kernel on kvs_retrieve's cap (16-byte data)
+    const uint32_t nhost = e_host - (uint32_t)ndev;
+    if (nhost) {
+        Job jh = j;
+        jh.entries = j.entries + ndev;
+        jh.entry_base = (uint32_t)ndev;
+        jh.num_entries = nhost;
+        jh.num_pieces = (uint64_t)nhost * P * bpc * ppr;
+        if (vec == 16)
+            NA_CUDA(launch_link(jh, cap ? cap : hostlink_grid(true), s));
+        else
+            NA_CUDA(launch_ldg(jh, vec, cap, s));
+    }
+    if (ndev) {
+        Job jd = j;
+        jd.entry_base = 0;
+        jd.num_entries = (uint32_t)ndev;
+        jd.num_pieces = ndev * P * bpc * ppr;
+        NA_CUDA(launch_ldg(jd, vec, cap, s));
+    }
     if (validate && any_demoted) {
-        j.blocks = (const int32_t*)(d + off_bc);
-        j.mode = MODE_COMPARE;
-        NA_CUDA(launch_ldg(j, vec, grid, s));
+        Job jc = j;
+        jc.blocks = (const int32_t*)(d + off_bc);
+        jc.entry_base = 0;
+        jc.num_entries = (uint32_t)nent;
+        jc.num_pieces = nent * P * bpc * ppr;
+        jc.mode = MODE_COMPARE;
+        NA_CUDA(launch_ldg(jc, vec, cap, s));
     }
     if (validate) {
         NA_CUDA(cudaMemcpyAsync(&g_err_host, d, sizeof(int32_t), cudaMemcpyDeviceToHost, s));
@@ -274,6 +337,15 @@ int retrieve_noalloc(const kvs_geometry* g, const kvs_paged_cache* cache, const 
 }
 
 }  // namespace
+
+void noalloc_forget_devices() {
+    std::lock_guard<std::mutex> lk(g_na_mu);
+    for (int d = 0; d < kMaxDevices; ++d) {
+        g_dev_ready[d] = false;
+        g_dev_addr[d] = nullptr;
+    }
+}
+
 }  // namespace kvs
 
 extern "C" int kvs_retrieve_noalloc(const kvs_geometry* geom, const kvs_paged_cache* cache,

@@ -26,9 +26,11 @@ int main(void) {
     CHECK(2, kvs_retrieve(NULL, &cache, NULL, 0, NULL, 0) == KVS_ERR_INVALID_ARG);
     CHECK(3, strlen(kvs_last_error()) > 0);
 
-    /* an empty call with a valid geometry needs no device */
+    /* an empty call with a valid geometry needs no device; the planes are live host
+     * buffers of the declared extent (8 blocks x 16 tokens x 4 heads x 64 dims x 2 B) */
     kvs_geometry g = {2, 4, 64, 2, 16, 256};
-    void* planes[4] = {(void*)0x1000, (void*)0x2000, (void*)0x3000, (void*)0x4000};
+    static unsigned char plane_mem[4][8 * 16 * 4 * 64 * 2];
+    void* planes[4] = {plane_mem[0], plane_mem[1], plane_mem[2], plane_mem[3]};
     cache.kv_planes = planes;
     cache.num_blocks = 8;
     CHECK(4, kvs_retrieve(&g, &cache, NULL, 0, NULL, 0) == KVS_OK);

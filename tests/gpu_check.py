@@ -105,3 +105,50 @@ def free(buf):
     buf.chunks = buf.store_chunks = []
     buf.requests = buf.store_requests = []
     torch.cuda.empty_cache()
+
+
+def random_workload(seed):
+    """Small seeded workload of random geometry: 1/2/4/8-byte elements, B in {1..32},
+    rows that are not a multiple of 16 bytes, ragged last chunks, non-zero first tokens,
+    mixed residency, and a stored suffix on some requests."""
+    rng = np.random.default_rng(seed)
+    e = int(rng.choice([1, 2, 2, 2, 4, 8]))
+    L = int(rng.integers(1, 5))
+    H = int(rng.integers(1, 9))
+    D = int(rng.choice([1, 3, 5, 8, 64, 128]))
+    B = int(rng.choice([1, 2, 8, 16, 32]))
+    C = B * int(rng.integers(1, 5))
+    nreq = int(rng.integers(1, 5))
+    prompts, matched, firsts, res, stores = [], [], [], [], []
+    for _ in range(nreq):
+        first = C * int(rng.integers(0, 2))
+        st = int(rng.integers(0, 2 * C + 1)) if rng.random() < 0.6 else 0
+        # a stored suffix starts where the match ends, so that end must be chunk-aligned
+        m = C * int(rng.integers(0, 5)) if st else int(rng.integers(0, 4 * C + 1))
+        prompts.append(first + m + st + int(rng.integers(0, B + 1)))
+        matched.append(m)
+        firsts.append(first)
+        res.append("device" if rng.random() < 0.4 else "host")
+        stores.append(st)
+    nb = sum(-(-p // B) for p in prompts) + int(rng.integers(0, 8))
+    return synth.custom(L, H, D, B, C, nb, prompts, matched, seed=seed, elem_bytes=e,
+                        residency=res, firsts=firsts, store_tokens=stores)
+
+
+def shared_workload(differ: bool):
+    """Three requests whose first two logical blocks name the same two physical blocks
+    (a shared prefix); with ``differ`` one token of the third request's copy differs."""
+    from paper_2609_35065_gb300 import buffers
+    g = synth.Geometry(2, 2, 8, 2, 4, 8)
+    perm = np.arange(40, dtype=np.int32)[::-1].copy()
+    t0 = perm[:6]
+    t1 = np.concatenate([t0[:2], perm[6:10]]).astype(np.int32)
+    t2 = np.concatenate([t0[:2], perm[10:12]]).astype(np.int32)
+    reqs = [synth.Request(24, 24, t0, "host", shared_prefix_tokens=0),
+            synth.Request(24, 24, t1, "device", shared_prefix_tokens=8),
+            synth.Request(16, 12, t2, "host", shared_prefix_tokens=8)]
+    w = synth.Workload("shared", g, 40, reqs, dist="uniform", seed=3)
+    buf = buffers.allocate(w)
+    if differ:
+        buf.chunks[2][0].view(4, 8, 16)[:, 1, :] += 1          # token 1 of request 2 differs
+    return buf

@@ -97,35 +97,9 @@ def test_tiny_device_resident_source(variant):
     gc.check_store(buf)
 
 
-def _random_workload(seed):
-    rng = np.random.default_rng(seed)
-    e = int(rng.choice([1, 2, 2, 2, 4, 8]))
-    L = int(rng.integers(1, 5))
-    H = int(rng.integers(1, 9))
-    D = int(rng.choice([1, 3, 5, 8, 64, 128]))
-    B = int(rng.choice([1, 2, 8, 16, 32]))
-    C = B * int(rng.integers(1, 5))
-    nreq = int(rng.integers(1, 5))
-    prompts, matched, firsts, res, stores = [], [], [], [], []
-    for _ in range(nreq):
-        first = C * int(rng.integers(0, 2))
-        st = int(rng.integers(0, 2 * C + 1)) if rng.random() < 0.6 else 0
-        # a stored suffix starts where the match ends, so that end must be chunk-aligned
-        m = C * int(rng.integers(0, 5)) if st else int(rng.integers(0, 4 * C + 1))
-        prompts.append(first + m + st + int(rng.integers(0, B + 1)))
-        matched.append(m)
-        firsts.append(first)
-        res.append("device" if rng.random() < 0.4 else "host")
-        stores.append(st)
-    nb = sum(-(-p // B) for p in prompts) + int(rng.integers(0, 8))
-    w = synth.custom(L, H, D, B, C, nb, prompts, matched, seed=seed, elem_bytes=e,
-                     residency=res, firsts=firsts, store_tokens=stores)
-    return w
-
-
 @pytest.mark.parametrize("seed", range(40))
 def test_random_small_geometries(seed):
-    w = _random_workload(seed)
+    w = gc.random_workload(seed)
     g = w.geom
     flags_all = [0, kvs.KVS_F_FORCE_HOSTLINK, kvs.KVS_F_FORCE_HBMCOPY, kvs.KVS_F_FORCE_LDG,
                  kvs.KVS_F_MAX_CTAS(1 + seed % 7)]
@@ -176,33 +150,16 @@ def test_tma_rejects_unaligned_rows():
     assert torch.all(buf.planes == buf.planes.view(-1)[0])     # nothing written
 
 
-def _shared(differ: bool):
-    # three requests whose first two blocks are shared physical blocks
-    g = synth.Geometry(2, 2, 8, 2, 4, 8)
-    perm = np.arange(40, dtype=np.int32)[::-1].copy()
-    t0 = perm[:6]
-    t1 = np.concatenate([t0[:2], perm[6:10]]).astype(np.int32)
-    t2 = np.concatenate([t0[:2], perm[10:12]]).astype(np.int32)
-    reqs = [synth.Request(24, 24, t0, "host", shared_prefix_tokens=0),
-            synth.Request(24, 24, t1, "device", shared_prefix_tokens=8),
-            synth.Request(16, 12, t2, "host", shared_prefix_tokens=8)]
-    w = synth.Workload("shared", g, 40, reqs, dist="uniform", seed=3)
-    buf = buffers.allocate(w)
-    if differ:
-        buf.chunks[2][0].view(4, 8, 16)[:, 1, :] += 1          # token 1 of request 2 differs
-    return buf
-
-
 @pytest.mark.parametrize("flags", [0, kvs.KVS_F_NO_DEDUP, kvs.KVS_F_FORCE_HBMCOPY])
 def test_shared_blocks_written_once_with_equal_content(flags):
-    buf = _shared(differ=False)
+    buf = gc.shared_workload(differ=False)
     _retrieve(buf, flags)
     torch.cuda.synchronize()
     gc.check_retrieve(buf)
 
 
 def test_shared_blocks_with_differing_bytes_are_reported():
-    buf = _shared(differ=True)
+    buf = gc.shared_workload(differ=True)
     with pytest.raises(kvs.KvsError) as ei:
         _retrieve(buf)
     assert ei.value.code == kvs.KVS_ERR_ALIAS

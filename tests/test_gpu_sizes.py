@@ -110,31 +110,55 @@ def test_qwen14b_store_to_hbm_destination_hbmcopy_path():
     gc.free(buf)
 
 
-def test_llama70b_quarter_buffer_refilled_between_passes():
-    """Pinned fast-tier buffer holds 25% of the batch: 4 passes, refilled in between."""
-    w = synth.llama70b(buffer_frac=0.25)
+@pytest.mark.parametrize("frac", [0.25, 0.5], ids=["25pct", "50pct"])
+def test_llama70b_partial_buffer_refilled_between_passes(frac):
+    """Pinned fast-tier buffer holds 25% (4 passes of one request) or 50% (2 passes of two
+    requests) of the batch, refilled in between; every pass is one call."""
+    w = synth.llama70b(buffer_frac=frac)
     g = w.geom
     per_tok = 2 * g.layers * g.row_elems
+    per_pass = int(round(len(w.requests) * frac))
     n = w.num_blocks * g.block_size * g.row_elems
     planes = torch.full((2 * g.layers, n), synth.SENTINEL_BF16, dtype=torch.int16, device="cuda")
+    ptrs = [int(planes[p].data_ptr()) for p in range(2 * g.layers)]
     one_req = w.requests[0].matched_tokens * per_tok
-    pinned = torch.empty(one_req, dtype=torch.int16, pin_memory=True)
-    assert pinned.numel() * 2 * len(w.requests) == w.matched_tokens * per_tok * 2
+    pinned = torch.empty(per_pass * one_req, dtype=torch.int16, pin_memory=True)
+    assert pinned.numel() * len(w.requests) == int(frac * len(w.requests)) * w.matched_tokens * per_tok
     host_copies = []
-    for k, r in enumerate(w.requests):
-        gen = torch.Generator(device="cuda").manual_seed(100 + k)
-        tmp = torch.empty(one_req, dtype=torch.int16, device="cuda")
-        synth.fill_values(tmp, "normal", gen)
+    for k in range(0, len(w.requests), per_pass):
+        tmp = torch.empty(per_pass * one_req, dtype=torch.int16, device="cuda")
+        synth.fill_values(tmp, "normal", torch.Generator(device="cuda").manual_seed(100 + k))
         torch.cuda.synchronize()
         pinned.copy_(tmp)                                   # refill between passes (untimed)
         del tmp
-        chunks = [pinned[j * 256 * per_tok:(j + 1) * 256 * per_tok] for j in range(r.matched_tokens // 256)]
-        req = kvs.RequestArg(r.block_table, [kvs.ChunkArg(c, 256) for c in chunks])
-        kvs.kvs_retrieve(g, [int(planes[p].data_ptr()) for p in range(2 * g.layers)], w.num_blocks,
-                         [req], None, kvs.KVS_F_VALIDATE)
+        reqs = []
+        for i, r in enumerate(w.requests[k:k + per_pass]):
+            base = i * one_req
+            chunks = [pinned[base + j * 256 * per_tok:base + (j + 1) * 256 * per_tok]
+                      for j in range(r.matched_tokens // 256)]
+            reqs.append(kvs.RequestArg(r.block_table, [kvs.ChunkArg(c, 256) for c in chunks]))
+            host_copies.append([c.numpy().copy().view(np.uint16) for c in chunks])
+        kvs.kvs_retrieve(g, ptrs, w.num_blocks, reqs, None, kvs.KVS_F_VALIDATE)
         torch.cuda.synchronize()
-        host_copies.append([c.numpy().copy().view(np.uint16) for c in chunks])
     fake = buffers.Buffers(w, planes, [], [], [], [])
     gc.check_retrieve(fake, chunks_np=host_copies)
     del planes, pinned
     torch.cuda.empty_cache()
+
+
+def test_llama70b_full_buffer_as_one_call():
+    """The 100% buffer: the whole 40 GiB batch (4 requests x 32,768 tokens, 512 chunks,
+    1,310,720 pieces of 32 KiB over 160 planes) in ONE call, in the launch configuration
+    the benchmark times (after kvs_query_bw, flags 0, a side stream); every element of
+    every plane against the oracle, one plane at a time."""
+    s = torch.cuda.Stream()
+    kvs.kvs_query_bw(s, 1 << 30)
+    w = synth.llama70b()
+    buf = buffers.allocate(w)
+    assert buf.payload_bytes == 40 << 30
+    assert sum(len(r.chunks) for r in buf.requests) * 2 * w.geom.layers * 16 == 1_310_720
+    kvs.kvs_retrieve(w.geom, buf.plane_ptrs, w.num_blocks, buf.requests, s, 0)
+    s.synchronize()
+    assert kvs.kvs_check_errors(s) == kvs.KVS_OK
+    gc.check_retrieve(buf)
+    gc.free(buf)
