@@ -29,17 +29,22 @@ import numpy as np
 
 _HERE = os.path.dirname(os.path.abspath(__file__))
 _SRC = os.path.join(_HERE, "kvs_oracle.c")
+_SRC_FP8 = os.path.join(_HERE, "kvs_oracle_fp8.c")
 _SO = os.path.join(_HERE, "_build", "libkvs_oracle.so")
 _lock = threading.Lock()
 _lib = None
 
 
 def build(force: bool = False) -> str:
-    """Compile ``kvs_oracle.c`` with gcc into ``oracle/_build`` (plain -O2, no tuning)."""
+    """Compile ``kvs_oracle.c`` and ``kvs_oracle_fp8.c`` with gcc into ``oracle/_build``
+    (plain -O2, no tuning; ISO C, so binary32 expressions are evaluated as written,
+    each operation rounded once, with no fused multiply-add)."""
     os.makedirs(os.path.dirname(_SO), exist_ok=True)
-    if force or not os.path.exists(_SO) or os.path.getmtime(_SO) < os.path.getmtime(_SRC):
+    srcs = [_SRC, _SRC_FP8]
+    if force or not os.path.exists(_SO) or any(os.path.getmtime(_SO) < os.path.getmtime(x) for x in srcs):
         tmp = _SO + f".{os.getpid()}.tmp"
-        subprocess.run(["gcc", "-O2", "-std=c11", "-shared", "-fPIC", _SRC, "-o", tmp], check=True)
+        subprocess.run(["gcc", "-O2", "-std=c11", "-ffp-contract=off", "-shared", "-fPIC", *srcs,
+                        "-o", tmp, "-lm"], check=True)
         os.replace(tmp, _SO)
     return _SO
 
@@ -65,6 +70,24 @@ def _bind(lib):
         fn.restype = ctypes.c_int
     lib.kvs_oracle_fill.argtypes = [P, ctypes.c_int64, ctypes.c_int, P]
     lib.kvs_oracle_fill.restype = None
+    sig8 = [ctypes.c_int] * 4 + [P, ctypes.c_int64, ctypes.c_int, ctypes.c_int,
+                                 ctypes.c_int64, ctypes.c_int, P, P, P, ctypes.c_int64]
+    for name in ("kvs_oracle_retrieve_fp8", "kvs_oracle_store_fp8"):
+        fn = getattr(lib, name)
+        fn.argtypes = sig8
+        fn.restype = ctypes.c_int
+    lib.kvs_oracle_e4m3_value.argtypes = [ctypes.c_uint8]
+    lib.kvs_oracle_e4m3_value.restype = ctypes.c_float
+    lib.kvs_oracle_e4m3_code.argtypes = [ctypes.c_float]
+    lib.kvs_oracle_e4m3_code.restype = ctypes.c_uint8
+    lib.kvs_oracle_bf16_bits.argtypes = [ctypes.c_float]
+    lib.kvs_oracle_bf16_bits.restype = ctypes.c_uint16
+    lib.kvs_oracle_fp8_scale_bytes.argtypes = [ctypes.c_int, ctypes.c_int]
+    lib.kvs_oracle_fp8_scale_bytes.restype = ctypes.c_int64
+    for name in ("kvs_oracle_e4m3_encode_array", "kvs_oracle_e4m3_decode_array", "kvs_oracle_bf16_encode_array"):
+        fn = getattr(lib, name)
+        fn.argtypes = [P, P, ctypes.c_int64]
+        fn.restype = None
     return lib
 
 
@@ -162,3 +185,78 @@ def store_fancy(L, H, D, B, planes, first_token, chunks, block_table):
             for kv in range(2):
                 view[l, kv] = planes[2 * l + kv].reshape(-1, H * D)[slots[start:start + n]]
         start += n
+
+
+# ----------------------------------------------------------------------------
+# fp8 chunks (kvs_oracle_fp8.c): E4M3 codes of the OCP OFP8 specification,
+# revision 1.0, with one binary32 scale per (chunk, layer, K/V, head).
+# ----------------------------------------------------------------------------
+
+def fp8_scale_bytes(L: int, H: int, lib=None) -> int:
+    """Bytes of the scale block at the head of an fp8 chunk buffer."""
+    return int((lib or load()).kvs_oracle_fp8_scale_bytes(L, H))
+
+
+def fp8_chunk_bytes(L: int, H: int, D: int, n: int, lib=None) -> int:
+    """Bytes of an fp8 chunk buffer of n tokens: scale block + [L][2][n][H][D] codes."""
+    return fp8_scale_bytes(L, H, lib) + 2 * L * n * H * D
+
+
+def e4m3_encode(x: np.ndarray, lib=None) -> np.ndarray:
+    """E4M3 codes of float32 values (round to nearest even, saturating; NaN -> 0x7F)."""
+    x = np.ascontiguousarray(x, dtype=np.float32)
+    out = np.empty(x.shape, dtype=np.uint8)
+    (lib or load()).kvs_oracle_e4m3_encode_array(_ptr(x), _ptr(out), x.size)
+    return out
+
+
+def e4m3_decode(c: np.ndarray, lib=None) -> np.ndarray:
+    """float32 values of E4M3 codes (NaN for 0x7F / 0xFF)."""
+    c = np.ascontiguousarray(c, dtype=np.uint8)
+    out = np.empty(c.shape, dtype=np.float32)
+    (lib or load()).kvs_oracle_e4m3_decode_array(_ptr(c), _ptr(out), c.size)
+    return out
+
+
+def bf16_encode(x: np.ndarray, lib=None) -> np.ndarray:
+    """BF16 bit patterns of float32 values (round to nearest even; NaN -> 0x7FFF)."""
+    x = np.ascontiguousarray(x, dtype=np.float32)
+    out = np.empty(x.shape, dtype=np.uint16)
+    (lib or load()).kvs_oracle_bf16_encode_array(_ptr(x), _ptr(out), x.size)
+    return out
+
+
+def _call_fp8(name, L, H, D, B, planes, num_blocks, first_token, chunks, chunk_tokens, block_table,
+              p0, p1, lib):
+    lib = lib or load()
+    p1 = 2 * L if p1 is None else p1
+    for a in planes:
+        if a is not None and a.dtype != np.uint16:
+            raise ValueError("fp8 oracle planes hold BF16 bit patterns (uint16)")
+    for c in chunks:
+        if c.dtype != np.uint8:
+            raise ValueError("fp8 chunks are byte buffers (uint8)")
+    plane_ptrs = (ctypes.c_void_p * (2 * L))(*[_ptr(a) for a in planes])
+    chunk_ptrs = (ctypes.c_void_p * max(1, len(chunks)))(*[_ptr(c) for c in chunks])
+    ntok = (ctypes.c_int32 * max(1, len(chunks)))(*[int(n) for n in chunk_tokens])
+    for c, n in zip(chunks, chunk_tokens):
+        if c.size < fp8_chunk_bytes(L, H, D, n, lib):
+            raise ValueError("fp8 chunk buffer smaller than its scale block and codes")
+    bt = np.ascontiguousarray(block_table, dtype=np.int32)
+    return getattr(lib, name)(L, H, D, B, plane_ptrs, int(num_blocks), p0, p1, int(first_token),
+                              len(chunks), chunk_ptrs, ntok, bt.ctypes.data, bt.size)
+
+
+def retrieve_fp8(L, H, D, B, planes, num_blocks, first_token, chunks, chunk_tokens, block_table,
+                 p0=0, p1=None, lib=None) -> int:
+    """Dequantising retrieval of one request: fp8 chunks (uint8 buffers) -> BF16 planes
+    (uint16 arrays).  Returns 0, or -2 when a token has no valid block."""
+    return _call_fp8("kvs_oracle_retrieve_fp8", L, H, D, B, planes, num_blocks, first_token,
+                     chunks, chunk_tokens, block_table, p0, p1, lib)
+
+
+def store_fp8(L, H, D, B, planes, num_blocks, first_token, chunks, chunk_tokens, block_table,
+              p0=0, p1=None, lib=None) -> int:
+    """Quantising store-back of one request: BF16 planes -> fp8 chunks (written in place)."""
+    return _call_fp8("kvs_oracle_store_fp8", L, H, D, B, planes, num_blocks, first_token,
+                     chunks, chunk_tokens, block_table, p0, p1, lib)

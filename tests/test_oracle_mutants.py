@@ -13,6 +13,7 @@ import pytest
 import oracle
 
 SRC = os.path.join(os.path.dirname(oracle.__file__), "kvs_oracle.c")
+SRC_FP8 = os.path.join(os.path.dirname(oracle.__file__), "kvs_oracle_fp8.c")   # built beside it, unmutated
 TESTS = os.path.dirname(os.path.abspath(__file__))
 ROOT = os.path.dirname(TESTS)
 
@@ -62,7 +63,8 @@ def test_mutant_is_caught(tmp_path, name):
     c = tmp_path / f"{name}.c"
     so = tmp_path / f"{name}.so"
     c.write_text(_mutate(name))
-    subprocess.run(["gcc", "-O1", "-std=c11", "-shared", "-fPIC", str(c), "-o", str(so)], check=True)
+    subprocess.run(["gcc", "-O1", "-std=c11", "-shared", "-fPIC", str(c), SRC_FP8, "-o", str(so), "-lm"],
+                   check=True)
     code = CHILD.format(root=ROOT, tests=TESTS, so=str(so))
     r = subprocess.run([sys.executable, "-c", code], capture_output=True, text=True, timeout=300)
     caught = r.returncode != 0 or ("FAILED:" in r.stdout and r.stdout.strip().split("FAILED:")[-1] != "")
@@ -72,7 +74,7 @@ def test_mutant_is_caught(tmp_path, name):
 def test_unmutated_copy_passes(tmp_path):
     """Control: the same harness on an unmodified copy reports no failure."""
     so = tmp_path / "clean.so"
-    subprocess.run(["gcc", "-O1", "-std=c11", "-shared", "-fPIC", SRC, "-o", str(so)], check=True)
+    subprocess.run(["gcc", "-O1", "-std=c11", "-shared", "-fPIC", SRC, SRC_FP8, "-o", str(so), "-lm"], check=True)
     code = CHILD.format(root=ROOT, tests=TESTS, so=str(so))
     r = subprocess.run([sys.executable, "-c", code], capture_output=True, text=True, timeout=300)
     assert r.returncode == 0 and r.stdout.strip().endswith("FAILED:"), r.stdout + r.stderr
