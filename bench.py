@@ -61,6 +61,8 @@ def parse_args(argv=None):
                     help="llama8b: retrieval (host->GPU) and store-back (GPU->host) at the same time")
     ap.add_argument("--side-priority", choices=["normal", "high"], default="high",
                     help="priority of the retrieval stream in --overlap runs")
+    ap.add_argument("--fp8", action="store_true",
+                    help="the workload's chunks as fp8 (E4M3 + per-head scales): retrieve and store-back rates")
     ap.add_argument("--no-extras", action="store_true",
                     help="default line without its extra legs (no-alloc, store to host, sweep50, overlap)")
     return ap.parse_args(argv)
@@ -847,13 +849,108 @@ def default_line_legs(args, buf, bw, stream, sampler, flags):
     del sb
     torch.cuda.empty_cache()
 
+    # fp8 chunks (E4M3 + per-head scales) of the same batch: half the bytes over the link
+    import copy
+    w8 = copy.deepcopy(w)
+    for r in w8.requests:                   # store the retrieved tokens back into fresh fp8 chunks
+        r.store_tokens, r.store_first = r.matched_tokens, r.first_token
+    fb = buffers.allocate_fp8(w8, store=True, with_planes=False)
+    fbytes = fb.payload_bytes
+    kvs.kvs_retrieve_fp8(g, buf.plane_ptrs, w.num_blocks, fb.requests, stream, kvs.KVS_F_VALIDATE)
+    sec, best, win = timed(lambda: kvs.kvs_retrieve_fp8(g, buf.plane_ptrs, w.num_blocks, fb.requests, stream, 0))
+    kvs.kvs_store_fp8(g, buf.plane_ptrs, w.num_blocks, fb.store_requests, stream, kvs.KVS_F_VALIDATE)
+    ssec, sbest, swin = timed(lambda: kvs.kvs_store_fp8(g, buf.plane_ptrs, w.num_blocks, fb.store_requests,
+                                                        stream, 0))
+    legs["fp8"] = {"retrieve": {"link_gbs": round(fbytes / sec / 1e9, 2),
+                                "frac_of_host_link": round(fbytes / sec / 1e9 / host_peak, 4),
+                                "tokens_per_s": round(w.matched_tokens / sec, 1),
+                                "bf16_bytes_delivered_gbs": round(payload / sec / 1e9, 2),
+                                "kernel": "kvs_fp8_retrieve_kernel", "clocks": sampler.summary(*win)},
+                   "store": {"link_gbs": round(fbytes / ssec / 1e9, 2),
+                             "frac_of_d2h_link": round(fbytes / ssec / 1e9 / d2h_peak, 4),
+                             "tokens_per_s": round(w.matched_tokens / ssec, 1),
+                             "kernel": "kvs_fp8_store_kernel", "clocks": sampler.summary(*swin)},
+                   "chunk_bytes": fbytes, "format": "OCP OFP8 rev 1.0 E4M3 codes + binary32 scale per "
+                                                    "(chunk, layer, K/V, head)", "calls": n}
+    del fb
+    torch.cuda.empty_cache()
+
     # retrieval beside a bf16 GEMM loop (70B shape, 25% buffer), default cap
     side = torch.cuda.Stream(priority=-1)
     w70 = synth.llama70b(buffer_frac=0.25)
-    results, info = overlap_measure(w70, bw, side, [("default", 0)], sampler)
+    results, info = overlap_measure(w70, bw, side, [("default", 0), ("dma", kvs.KVS_F_FORCE_DMA)], sampler)
     legs["overlap"] = {"workload": describe(w70), **info, "hostlink_ctas": kvs.kvs_get_choice()["hostlink_ctas"],
                        "side_stream": "high priority", **results}
     return legs
+
+
+def run_fp8(args):
+    """Retrieval from, and store-back into, fp8 chunks (E4M3 codes with one binary32 scale
+    per chunk, layer, K/V and head) of the workload, host-resident as in its config:
+    link GB/s (fp8 bytes), prefix tokens/s, and the BF16 line's tokens/s for comparison."""
+    import copy
+    import torch
+    from paper_2609_35065_gb300 import buffers, kvs
+
+    torch.cuda.set_device(0)
+    kvs.lib()
+    stream = torch.cuda.Stream()
+    bw = kvs.kvs_get_choice() if args.skip_probe else kvs.kvs_query_bw(stream, args.probe_bytes)
+    host_peak = max(bw["h2d_copy_engine_gbs"], bw["zero_copy_read_gbs"]) or float("nan")
+    d2h_peak = max(bw["d2h_copy_engine_gbs"], bw["zero_copy_write_gbs"]) or float("nan")
+    w = copy.deepcopy(workload(args.config))
+    for r in w.requests:
+        r.store_tokens, r.store_first = r.matched_tokens, r.first_token
+    g = w.geom
+    fb = buffers.allocate_fp8(w, store=True)
+    fbytes = fb.payload_bytes
+    flags = kvs.KVS_F_MAX_CTAS(args.max_ctas) if args.max_ctas else 0
+
+    def timed(fn, k):
+        evs = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)) for _ in range(k)]
+        for a, b in evs:
+            a.record(stream)
+            fn()
+            b.record(stream)
+        torch.cuda.synchronize()
+        return [a.elapsed_time(b) / 1e3 for a, b in evs]
+
+    def ret():
+        kvs.kvs_retrieve_fp8(g, fb.plane_ptrs, w.num_blocks, fb.requests, stream, flags)
+
+    def sto():
+        kvs.kvs_store_fp8(g, fb.plane_ptrs, w.num_blocks, fb.store_requests, stream, flags)
+
+    kvs.kvs_retrieve_fp8(g, fb.plane_ptrs, w.num_blocks, fb.requests, stream, flags | kvs.KVS_F_VALIDATE)
+    kvs.kvs_store_fp8(g, fb.plane_ptrs, w.num_blocks, fb.store_requests, stream, flags | kvs.KVS_F_VALIDATE)
+    for _ in range(args.warmup):
+        ret()
+        sto()
+    torch.cuda.synchronize()
+    sampler = ClockSampler(torch.cuda.current_device())
+    time.sleep(0.15)
+    t0 = time.time()
+    rs = timed(ret, args.steps)
+    t1 = time.time()
+    ss = timed(sto, args.steps)
+    t2 = time.time()
+    time.sleep(0.1)
+    sampler.stop()
+    rm, sm = statistics.mean(rs), statistics.mean(ss)
+    line = {"metric": METRIC + " (fp8 chunks)", "unit": "GB/s", "value": round(fbytes / rm / 1e9, 3),
+            "steps": args.steps, "warmup": args.warmup, "dtype": "fp8 e4m3 chunks -> bf16 planes",
+            "config": {"workload": describe(w), "source": "pinned host memory" if w.requests[0].residency == "host"
+                       else "HBM", "chunk_bytes": fbytes,
+                       "format": "OCP OFP8 rev 1.0 E4M3 + binary32 scale per (chunk, layer, K/V, head)"},
+            "retrieve": {"link_gbs": round(fbytes / rm / 1e9, 2), "frac_of_host_link": round(fbytes / rm / 1e9 / host_peak, 4),
+                         "tokens_per_s": round(w.matched_tokens / rm, 1), "ms": round(rm * 1e3, 4),
+                         "clocks": sampler.summary(t0, t1)},
+            "store": {"link_gbs": round(fbytes / sm / 1e9, 2), "frac_of_d2h_link": round(fbytes / sm / 1e9 / d2h_peak, 4),
+                      "tokens_per_s": round(w.matched_tokens / sm, 1), "ms": round(sm * 1e3, 4),
+                      "clocks": sampler.summary(t1, t2)},
+            "host_link_peak_gbs": round(host_peak, 2), "d2h_link_peak_gbs": round(d2h_peak, 2)}
+    print(json.dumps(line), flush=True)
+    return 0
 
 
 def run_overlap(args):
@@ -873,6 +970,7 @@ def run_overlap(args):
                 ("hostlink_12ctas", kvs.KVS_F_FORCE_HOSTLINK | kvs.KVS_F_MAX_CTAS(12)),
                 ("hostlink_24ctas", kvs.KVS_F_FORCE_HOSTLINK | kvs.KVS_F_MAX_CTAS(24)),
                 ("hbmcopy", kvs.KVS_F_FORCE_HBMCOPY),
+                ("dma", kvs.KVS_F_FORCE_DMA),
                 ("layer_launches", kvs.KVS_F_LAYER_LAUNCHES),
                 ("layer_launches_96ctas", kvs.KVS_F_LAYER_LAUNCHES | kvs.KVS_F_MAX_CTAS(96))]
     sampler = ClockSampler(torch.cuda.current_device())
@@ -1361,6 +1459,8 @@ def main(argv=None):
         return run_reference(args)
     if args.overlap:
         return run_overlap(args)
+    if args.fp8:
+        return run_fp8(args)
     if args.layerwise:
         return run_layerwise(args)
     if args.duplex:

@@ -90,12 +90,19 @@ extern "C" {
                                           (the default; accepted for explicitness)         */
 #define KVS_F_LAYER_SIGNAL   (1u << 7) /* layer-wise calls: one resident launch that
                                           signals each group (see kvs_retrieve_layers)     */
+#define KVS_F_FORCE_DMA      (1u << 8) /* host chunks: the copy engine moves each (chunk,
+                                          block) straight between the chunk and all 2L
+                                          planes with one 2D copy; no SM runs a kernel for
+                                          them.  Needs equally spaced planes (plane p at
+                                          plane 0 + p * pitch, as in one [2L][...] cache
+                                          allocation); KVS_ERR_UNSUPPORTED otherwise      */
 #define KVS_F_MAX_CTAS(n)    ((((uint32_t)(n)) & 0xFFFFu) << 16) /* cap on CTAs, 0 = auto */
 #define KVS_F_GET_MAX_CTAS(f) (((f) >> 16) & 0xFFFFu)
 
 /* Variant identifiers reported by kvs_query_bw. */
 #define KVS_VARIANT_HOSTLINK 1
 #define KVS_VARIANT_HBMCOPY  2
+#define KVS_VARIANT_DMA      3
 #define KVS_KERNEL_LDG       1
 #define KVS_KERNEL_TMA       2
 
@@ -211,6 +218,49 @@ int kvs_store_layers(const kvs_geometry* geom, const kvs_paged_cache* cache,
                      int32_t layers_per_step, void* const* ready_events,
                      void* const* layer_events, void* cuda_stream, uint32_t flags);
 
+/*
+ * fp8 chunks.  The paper keeps KV in BF16 (Sec. 5 setup) and retains it in
+ * 256-token chunks (Sec. 5.1, Workload); these two calls add a compressed
+ * chunk format for the fast tier, which halves the bytes a retrieval moves
+ * over the host link.  A chunk of n tokens is one buffer:
+ *
+ *   [scales] 2L*H IEEE binary32 values, the scale of (layer l, K/V kv, head h)
+ *            at index (2l + kv)*H + h, zero-padded to KVS_FP8_SCALE_BYTES(L, H)
+ *            bytes (a multiple of 256);
+ *   [codes]  [L][2][n][H][D] bytes in the E4M3 format of the OCP 8-bit
+ *            Floating Point Specification (OFP8), revision 1.0.
+ *
+ * The paged planes stay BF16 (geom->elem_bytes must be 2).  head_dim must be
+ * a multiple of 16, H at most 128, chunks and planes 16-byte aligned
+ * (KVS_ERR_UNSUPPORTED otherwise).  Arguments, layouts of the planes and
+ * block tables, residencies, asynchrony and errors are as for kvs_retrieve /
+ * kvs_store; the accepted flags are KVS_F_VALIDATE, KVS_F_MAX_CTAS (and
+ * KVS_F_FORCE_HOSTLINK / KVS_F_FORCE_LDG, which name what always runs: host
+ * chunks are read or written over the host link by SM loads and stores).
+ *
+ * kvs_retrieve_fp8: plane[2l+kv][slot(s_j+i)][h][d] =
+ *     bf16(e4m3(code[l][kv][i][h][d]) * scale[l][kv][h]): the product is one
+ *     binary32 multiply rounded to nearest even, then rounded to BF16 (nearest
+ *     even); a NaN product (a NaN code, or a NaN scale) gives 0x7FFF.  A
+ *     physical block named by two requests of one call is refused
+ *     (KVS_ERR_ALIAS): quantised copies of one block differ with the scales of
+ *     the chunks that hold them.
+ * kvs_store_fp8: for every chunk, layer, K/V and head, amax = the largest |x|
+ *     over the finite BF16 elements of the chunk's tokens (0 if none), scale =
+ *     amax / 448 (binary32, nearest even; 1 when amax is 0), code = E4M3 of
+ *     x / scale (binary32 division, nearest even), rounded to nearest even
+ *     and saturated to +-448 (OFP8 saturation mode; infinities too); NaN
+ *     elements give the code 0x7F.  The scales and codes of every destination
+ *     chunk are written; the cache is only read.
+ */
+#define KVS_FP8_SCALE_BYTES(L, H) ((((int64_t)2 * (L) * (H) * 4) + 255) / 256 * 256)
+int kvs_retrieve_fp8(const kvs_geometry* geom, const kvs_paged_cache* cache,
+                     const kvs_request* requests, int32_t num_requests,
+                     void* cuda_stream, uint32_t flags);
+int kvs_store_fp8(const kvs_geometry* geom, const kvs_paged_cache* cache,
+                  const kvs_request* requests, int32_t num_requests,
+                  void* cuda_stream, uint32_t flags);
+
 /* Bandwidths measured by kvs_query_bw, in GB/s (1e9 bytes per second). */
 typedef struct kvs_bw_report {
     double  hbm_copy_gbs;          /* device->device copy kernel, read + write bytes      */
@@ -231,6 +281,8 @@ typedef struct kvs_bw_report {
                                       (before any kvs_query_bw: one per 3 SMs)            */
     int32_t store_ctas;            /* the same for host-link store kernels                 */
     int64_t probe_bytes;           /* bytes moved per probe                                */
+    double  retrieve_dma_gbs;      /* host-chunk retrieval probe, DMA variant              */
+    double  store_dma_gbs;         /* host-chunk store probe, DMA variant                  */
 } kvs_bw_report;
 
 /*
@@ -246,6 +298,37 @@ int kvs_query_bw(kvs_bw_report* out, void* cuda_stream, int64_t probe_bytes);
 /* Reads the defaults currently in force on this device (after kvs_query_bw,
  * or the built-in ones) into `out`; bandwidth fields are 0 if never measured. */
 int kvs_get_choice(kvs_bw_report* out);
+
+/*
+ * Variant choice measured on the caller's own call.  kvs_query_bw probes a
+ * fixed 1 GiB pattern; how fast the copy engine moves host memory can depend
+ * on the buffer (its size and how it was allocated) and on what else the GPU
+ * runs, which only the real call shows.  kvs_tune performs the given call
+ * (direction KVS_DIR_RETRIEVE or KVS_DIR_STORE) `reps` + 1 times with each
+ * variant that can serve its host-resident chunks -- HOSTLINK, HBMCOPY and,
+ * with equally spaced planes, DMA -- times each on cuda_stream (best of
+ * `reps`, after one untimed run), and makes the fastest the default of later
+ * kvs_retrieve / kvs_store calls in that direction on this device.  Every
+ * candidate produces the same result, so the call's copy is done when
+ * kvs_tune returns (the stream is synchronised).  KVS_F_MAX_CTAS(n) caps the
+ * HOSTLINK candidate's grid (and becomes the host-link cap of that direction
+ * if it wins); KVS_F_VALIDATE is honoured on the untimed runs; FORCE flags are
+ * KVS_ERR_INVALID_ARG.  A call with no host-resident chunk changes nothing.
+ * `out` (may be NULL) receives the rates in GB/s of host-chunk bytes (0 for a
+ * candidate that cannot serve the call) and the choice.
+ */
+#define KVS_DIR_RETRIEVE 0
+#define KVS_DIR_STORE    1
+typedef struct kvs_tune_report {
+    double  gbs[3];            /* [HOSTLINK, HBMCOPY, DMA]                              */
+    int64_t host_bytes;        /* bytes of host-resident chunks in the call             */
+    int32_t chosen;            /* KVS_VARIANT_* now the default for this direction      */
+    int32_t direction;         /* KVS_DIR_*                                             */
+} kvs_tune_report;
+int kvs_tune(const kvs_geometry* geom, const kvs_paged_cache* cache,
+             const kvs_request* requests, int32_t num_requests,
+             void* cuda_stream, uint32_t flags, int32_t direction, int32_t reps,
+             kvs_tune_report* out);
 
 /*
  * Synchronises cuda_stream, then reads and clears this device's error word.
@@ -428,7 +511,7 @@ void* kvs_tier_slot(const kvs_tier* tier, int64_t slot);
 
 /* ABI version of this header: major * 10000 + minor * 100 + patch. */
 int kvs_version(void);
-#define KVS_VERSION 10600
+#define KVS_VERSION 10800
 
 #ifdef __cplusplus
 }

@@ -180,3 +180,115 @@ def allocate(w: synth.Workload, device: str = "cuda", store: bool = False,
         torch.cuda.synchronize()
     return Buffers(w, planes, chunks, store_chunks, requests, store_requests,
                    host_pool, device_pool, store_pool, plane_init)
+
+
+# ----------------------------------------------------------------------------
+# fp8 chunks: [scale block][E4M3 codes]
+# ----------------------------------------------------------------------------
+
+def fp8_chunk_bytes(g: synth.Geometry, n: int) -> int:
+    """Bytes of an fp8 chunk of n tokens: the 2L*H binary32 scale block padded to a
+    multiple of 256 bytes, then [L][2][n][H][D] one-byte codes."""
+    scale = (2 * g.layers * g.kv_heads * 4 + 255) // 256 * 256
+    return scale + 2 * g.layers * n * g.kv_heads * g.head_dim
+
+
+@dataclass
+class Fp8Buffers:
+    workload: synth.Workload
+    planes: torch.Tensor | None                    # [2L, NB*B*H*D] BF16 bit patterns (int16), cuda
+    chunks: list[list[torch.Tensor]]               # per request: fp8 chunk buffers (uint8)
+    store_chunks: list[list[torch.Tensor]]         # per request: fp8 destinations of the stored suffix
+    requests: list[RequestArg]
+    store_requests: list[RequestArg]
+    pools: list = field(default_factory=list)
+
+    plane_ptrs = Buffers.plane_ptrs
+    _ptrs: tuple = (None, None)
+
+    @property
+    def payload_bytes(self) -> int:
+        """Bytes of the retrieved fp8 chunks (scale blocks and codes)."""
+        return sum(int(t.numel()) for mine in self.chunks for t in mine)
+
+    def initial_plane(self, p: int) -> np.ndarray:
+        g = self.workload.geom
+        return np.full(self.workload.num_blocks * g.block_size * g.row_elems, synth.SENTINEL_BF16, dtype=np.uint16)
+
+
+def _fp8_pool(w, counts, residency, device, pin):
+    """One pool holding chunks of the given token counts at 256-byte aligned offsets."""
+    sizes = [fp8_chunk_bytes(w.geom, n) for n in counts]
+    offs, at = [], 0
+    for s in sizes:
+        offs.append(at)
+        at += (s + 255) // 256 * 256
+    if residency == "host":
+        pool = torch.zeros(max(at, 1), dtype=torch.uint8, pin_memory=pin)
+    else:
+        pool = torch.zeros(max(at, 1), dtype=torch.uint8, device=device)
+    return pool, [pool[o:o + s] for o, s in zip(offs, sizes)]
+
+
+def fill_fp8_chunk(t: torch.Tensor, g: synth.Geometry, gen: torch.Generator) -> None:
+    """Seeded fp8 chunk content: 2L*H positive binary32 scales in [2^-9, 2^-5) (the
+    range amax / 448 takes for KV of unit scale) and uniformly random code bytes (NaN
+    codes included, at their natural rate of 2 in 256)."""
+    ns = 2 * g.layers * g.kv_heads
+    dev = gen.device
+    sc = (torch.rand(ns, generator=gen, device=dev, dtype=torch.float32) * 4 + 1) * (2.0 ** -9)
+    codes = torch.randint(0, 256, (t.numel() - ((ns * 4 + 255) // 256 * 256),), generator=gen, device=dev,
+                          dtype=torch.int16).to(torch.uint8)
+    t[:ns * 4].copy_(sc.view(torch.uint8).to(t.device))
+    t[(ns * 4 + 255) // 256 * 256:].copy_(codes.to(t.device))
+
+
+def allocate_fp8(w: synth.Workload, device: str = "cuda", store: bool = False,
+                 store_residency: str = "host", with_planes: bool = True) -> Fp8Buffers:
+    """Sentinel-filled BF16 planes, seeded fp8 chunks for every request's matched prefix
+    (pinned host or HBM, per request), and, with ``store``, zeroed fp8 destinations for
+    each request's ``store_tokens`` suffix."""
+    g = w.geom
+    pin = torch.device(device).type == "cuda"
+    gen = torch.Generator(device=device).manual_seed(w.seed)
+    planes = None
+    if with_planes:
+        n = w.num_blocks * g.block_size * g.row_elems
+        sent = int(np.array([synth.SENTINEL_BF16], dtype=np.uint16).view(np.int16)[0])
+        planes = torch.full((2 * g.layers, n), sent, dtype=torch.int16, device=device)
+    pools, requests, views = [], [], {}
+    for res in ("host", "device"):
+        counts = [n for r in w.requests if r.residency == res for n in w.chunk_counts(r)]
+        if counts:
+            pool, v = _fp8_pool(w, counts, res, device, pin)
+            pools.append(pool)
+            views[res] = iter(v)
+    chunk_lists = []
+    for r in w.requests:
+        mine = [next(views[r.residency]) for _ in w.chunk_counts(r)]
+        for t in mine:
+            fill_fp8_chunk(t, g, gen)
+        res = KVS_SRC_HOST_PINNED if r.residency == "host" else KVS_SRC_DEVICE
+        requests.append(RequestArg(r.block_table, [ChunkArg(t, n, res) for t, n in zip(mine, w.chunk_counts(r))],
+                                   first_token=r.first_token))
+        chunk_lists.append(mine)
+    store_chunks, store_requests = [], []
+    if store:
+        counts = [n for r in w.requests for n in w.chunk_counts(r, r.store_tokens)]
+        if counts:
+            pool, views = _fp8_pool(w, counts, store_residency, device, pin)
+            pools.append(pool)
+            it = iter(views)
+            res = KVS_SRC_HOST_PINNED if store_residency == "host" else KVS_SRC_DEVICE
+            for r in w.requests:
+                cn = w.chunk_counts(r, r.store_tokens)
+                mine = [next(it) for _ in cn]
+                store_chunks.append(mine)
+                store_requests.append(RequestArg(r.block_table, [ChunkArg(t, n, res) for t, n in zip(mine, cn)],
+                                                 first_token=r.store_start if r.store_tokens else 0))
+        else:
+            store_chunks = [[] for _ in w.requests]
+            store_requests = [RequestArg(r.block_table, [], 0) for r in w.requests]
+    if torch.device(device).type == "cuda":
+        torch.cuda.synchronize()
+    return Fp8Buffers(w, planes, chunk_lists, store_chunks, requests, store_requests, pools)

@@ -13,7 +13,10 @@
 //                              host memory over the host link directly, or
 //                              HBMCOPY: the copy engine moves whole chunks
 //                              through a ring of HBM staging slots and the
-//                              device kernel scatters/gathers from there.
+//                              device kernel scatters/gathers from there, or
+//                              DMA: the copy engine scatters/gathers directly,
+//                              one 2D copy per (chunk, block) across all planes
+//                              (equally spaced planes only; no SMs used).
 #include <algorithm>
 #include <cstdarg>
 #include <cstdio>
@@ -109,6 +112,7 @@ struct DevState {
     int          retrieve_host = KVS_VARIANT_HOSTLINK;
     int          store_host = KVS_VARIANT_HOSTLINK;
     int          kernel_device = KVS_KERNEL_LDG;
+    size_t       max_pitch = 0;              // largest pitch a 2D copy accepts
     int          hostlink_ctas = 0;          // CTA cap of host-link kernels, 0 = whole GPU
     int          store_ctas = 0;
     kvs_bw_report report{};
@@ -126,6 +130,11 @@ int get_state(DevState** out) {
     if (!st.ready) {
         st.device = dev;
         KVS_CUDA(cudaDeviceGetAttribute(&st.sms, cudaDevAttrMultiProcessorCount, dev));
+        {
+            int mp = 0;
+            KVS_CUDA(cudaDeviceGetAttribute(&mp, cudaDevAttrMaxPitch, dev));
+            st.max_pitch = mp > 0 ? (size_t)mp : 0;
+        }
         KVS_CUDA(cudaMalloc(&st.err, sizeof(int32_t)));
         KVS_CUDA(cudaMemset(st.err, 0, sizeof(int32_t)));
         KVS_CUDA(cudaHostAlloc(&st.err_host, sizeof(int32_t), cudaHostAllocDefault));
@@ -282,8 +291,12 @@ int validate_call(const kvs_geometry* g, const kvs_paged_cache* cache,
 // exactly when some earlier span ends after it starts, so one sweep keeping
 // the furthest end (over all spans and over written spans) finds every
 // conflicting pair's later member.  Host only: no device work.
+uint64_t fp8_scale_bytes(const kvs_geometry* g) {
+    return ((uint64_t)2 * g->num_layers * g->num_kv_heads * 4 + 255) / 256 * 256;
+}
+
 int check_overlaps(const kvs_geometry* g, const kvs_paged_cache* cache, const kvs_request* reqs,
-                   int32_t nreq, bool retrieve) {
+                   int32_t nreq, bool retrieve, bool fp8 = false) {
     struct Span {
         uint64_t lo, hi;
         bool plane;
@@ -301,7 +314,9 @@ int check_overlaps(const kvs_geometry* g, const kvs_paged_cache* cache, const kv
         for (int32_t j = 0; j < reqs[r].num_chunks; ++j) {
             const kvs_chunk& c = reqs[r].chunks[j];
             const uint64_t lo = (uint64_t)c.base;
-            sp.push_back({lo, lo + (uint64_t)P * c.num_tokens * row, false, r, j});
+            const uint64_t bytes = fp8 ? fp8_scale_bytes(g) + (uint64_t)P * c.num_tokens * row / 2
+                                       : (uint64_t)P * c.num_tokens * row;
+            sp.push_back({lo, lo + bytes, false, r, j});
         }
     std::sort(sp.begin(), sp.end(), [](const Span& x, const Span& y) { return x.lo < y.lo; });
     auto name = [](const Span& x) {
@@ -617,6 +632,48 @@ int run_hbmcopy(DevState& st, const kvs_geometry* g, const kvs_paged_cache* cach
     return KVS_OK;
 }
 
+// Spacing of the planes when plane p starts at plane 0 + p * pitch for every p
+// (one [2L][NB*B*H*D] allocation), with the pitch within the 2D-copy limit;
+// 0 otherwise.
+uint64_t dma_pitch(const DevState& st, const Plan& pl, uint64_t row_span) {
+    const size_t P = pl.planes.size();
+    if (P < 2) return row_span;
+    if (pl.planes[1] <= pl.planes[0]) return 0;
+    const uint64_t pitch = pl.planes[1] - pl.planes[0];
+    if (pitch < row_span || pitch > st.max_pitch) return 0;
+    for (size_t p = 2; p < P; ++p)
+        if (pl.planes[p] != pl.planes[0] + p * pitch) return 0;
+    return pitch;
+}
+
+// Host chunks by the copy engine alone: for each (chunk, block) one 2D copy
+// whose rows are the 2L planes -- source rows n*R apart in the chunk,
+// destination rows `pitch` apart in the cache -- each row the block's tokens
+// x R bytes.  Blocks dropped by de-duplication are skipped.  No kernel runs.
+int run_dma(const kvs_geometry* g, const Plan& pl, uint64_t pitch, bool retrieve, cudaStream_t s,
+            const std::vector<const void*>& host_addr) {
+    const int B = g->block_size;
+    const size_t P = pl.planes.size();
+    const uint64_t R = pl.row_bytes;
+    for (uint32_t e = pl.num_device; e < pl.entries.size(); ++e) {
+        const int32_t n = pl.entries[e].n_tok;
+        const uint8_t* chunk = (const uint8_t*)host_addr[e - pl.num_device];
+        for (uint32_t i = 0; i < pl.bpc && (int32_t)i * B < n; ++i) {
+            const int32_t blk = pl.blocks[(size_t)e * pl.bpc + i];
+            if (blk < 0) continue;
+            const uint64_t width = (uint64_t)std::min(B, n - (int32_t)i * B) * R;
+            uint8_t* c = (uint8_t*)chunk + (uint64_t)i * B * R;
+            uint8_t* q = (uint8_t*)pl.planes[0] + (uint64_t)blk * B * R;
+            cudaError_t err = retrieve
+                ? cudaMemcpy2DAsync(q, pitch, c, (uint64_t)n * R, width, P, cudaMemcpyDefault, s)
+                : cudaMemcpy2DAsync(c, (uint64_t)n * R, q, pitch, width, P, cudaMemcpyDefault, s);
+            if (err != cudaSuccess)
+                return fail(KVS_ERR_CUDA, "2D copy of chunk %u block %u failed: %s", e, i, cudaGetErrorString(err));
+        }
+    }
+    return KVS_OK;
+}
+
 int read_error_word(DevState& st, cudaStream_t s) {
     KVS_CUDA(cudaMemcpyAsync(st.err_host, st.err, sizeof(int32_t), cudaMemcpyDeviceToHost, s));
     KVS_CUDA(cudaStreamSynchronize(s));
@@ -639,15 +696,16 @@ int copy_call(const kvs_geometry* g, const kvs_paged_cache* cache, const kvs_req
               int32_t layers_per_step = 0, void* const* layer_events = nullptr,
               void* const* ready_events = nullptr) {
     const bool f_host = flags & KVS_F_FORCE_HOSTLINK, f_hbm = flags & KVS_F_FORCE_HBMCOPY;
+    const bool f_dma = flags & KVS_F_FORCE_DMA;
     const bool f_ldg = flags & KVS_F_FORCE_LDG, f_tma = flags & KVS_F_FORCE_TMA;
-    if ((f_host && f_hbm) || (f_ldg && f_tma))
+    if ((int)f_host + (int)f_hbm + (int)f_dma > 1 || (f_ldg && f_tma))
         return fail(KVS_ERR_INVALID_ARG, "conflicting FORCE flags");
     if ((flags & KVS_F_LAYER_LAUNCHES) && (flags & KVS_F_LAYER_SIGNAL))
         return fail(KVS_ERR_INVALID_ARG, "KVS_F_LAYER_LAUNCHES and KVS_F_LAYER_SIGNAL together");
     if (ready_events && (flags & KVS_F_LAYER_SIGNAL))
         return fail(KVS_ERR_INVALID_ARG, "ready events need one launch per group, not KVS_F_LAYER_SIGNAL");
     if (layers_per_step < 0) return fail(KVS_ERR_INVALID_ARG, "layers_per_step must be positive");
-    if (layers_per_step > 0 && f_hbm)
+    if (layers_per_step > 0 && (f_hbm || f_dma))
         return fail(KVS_ERR_UNSUPPORTED, "layer-wise copies move host chunks over the host link only");
     Plan pl;
     int rc = validate_call(g, cache, reqs, nreq, pl);
@@ -680,9 +738,18 @@ int copy_call(const kvs_geometry* g, const kvs_paged_cache* cache, const kvs_req
         if (f_tma) return fail(KVS_ERR_UNSUPPORTED, "TMA needs 16-byte aligned chunks, planes and rows");
         flavour = KVS_KERNEL_LDG;
     }
-    int host_variant = f_host ? KVS_VARIANT_HOSTLINK : f_hbm ? KVS_VARIANT_HBMCOPY
+    int host_variant = f_host ? KVS_VARIANT_HOSTLINK : f_hbm ? KVS_VARIANT_HBMCOPY : f_dma ? KVS_VARIANT_DMA
                                                             : (retrieve ? st.retrieve_host : st.store_host);
     if (layers_per_step > 0) host_variant = KVS_VARIANT_HOSTLINK;
+    uint64_t pitch = 0;
+    if (host_variant == KVS_VARIANT_DMA && pl.num_host) {
+        pitch = dma_pitch(st, pl, (uint64_t)g->block_size * pl.row_bytes);
+        if (!pitch) {
+            if (f_dma) return fail(KVS_ERR_UNSUPPORTED, "KVS_F_FORCE_DMA needs equally spaced planes "
+                                   "(plane p at plane 0 + p * pitch, pitch within the 2D-copy limit)");
+            host_variant = KVS_VARIANT_HOSTLINK;
+        }
+    }
     const Mode mode = retrieve ? MODE_RETRIEVE : MODE_STORE;
     const int host_grid = grid ? grid : (retrieve ? st.hostlink_ctas : st.store_ctas);
 
@@ -761,11 +828,12 @@ int copy_call(const kvs_geometry* g, const kvs_paged_cache* cache, const kvs_req
             KVS_CUDA(cudaStreamWaitEvent(st.aux_stream, st.ev_aux_fork, 0));
         }
         if (pl.num_host) {
-            if (host_variant == KVS_VARIANT_HBMCOPY) {
+            if (host_variant == KVS_VARIANT_HBMCOPY || host_variant == KVS_VARIANT_DMA) {
                 std::vector<const void*> host_addr(pl.num_host);
                 for (uint32_t e = pl.num_device; e < pl.entries.size(); ++e)
                     host_addr[e - pl.num_device] = (const void*)pl.entries[e].chunk;
-                rc = run_hbmcopy(st, g, cache, pl, u, mode, flavour, grid, s, host_addr);
+                rc = host_variant == KVS_VARIANT_DMA ? run_dma(g, pl, pitch, retrieve, s, host_addr)
+                                                     : run_hbmcopy(st, g, cache, pl, u, mode, flavour, grid, s, host_addr);
             } else {
                 rc = launch_kernel(make_job(st, g, cache, pl, u, pl.num_device, pl.num_host, mode, p0, np),
                                    kKernelLink, vec, host_grid, s);
@@ -790,6 +858,98 @@ int copy_call(const kvs_geometry* g, const kvs_paged_cache* cache, const kvs_req
     }
     if (flags & KVS_F_VALIDATE) {
         KVS_CUDA(cudaEventRecord(u.slot->done, s));       // before the synchronising read
+        u.slot->used = true;
+        guard.slot = nullptr;
+        return read_error_word(st, s);
+    }
+    return KVS_OK;
+}
+
+// fp8 chunks (E4M3 codes with per-head binary32 scales) <-> BF16 planes.  Host
+// chunks run first on the host-link grid, device chunks after them on the
+// same stream.  A physical block named by two requests is refused: the
+// quantised copies of a shared block differ with each chunk's scales, so no
+// single writer would be the right one.
+int fp8_call(const kvs_geometry* g, const kvs_paged_cache* cache, const kvs_request* reqs,
+             int32_t nreq, void* stream, uint32_t flags, bool retrieve) {
+    const uint32_t allowed = KVS_F_VALIDATE | KVS_F_FORCE_HOSTLINK | KVS_F_FORCE_LDG | 0xFFFF0000u;
+    if (flags & ~allowed)
+        return fail(KVS_ERR_UNSUPPORTED, "fp8 calls take only KVS_F_VALIDATE, KVS_F_FORCE_HOSTLINK, "
+                    "KVS_F_FORCE_LDG and KVS_F_MAX_CTAS");
+    Plan pl;
+    int rc = validate_call(g, cache, reqs, nreq, pl);
+    if (rc) return rc;
+    if (g->elem_bytes != 2)
+        return fail(KVS_ERR_INVALID_ARG, "fp8 chunks fill BF16 planes: elem_bytes must be 2 (got %d)", g->elem_bytes);
+    if (g->head_dim % 16)
+        return fail(KVS_ERR_UNSUPPORTED, "fp8 chunks need head_dim a multiple of 16 (got %d)", g->head_dim);
+    if ((uint32_t)g->num_kv_heads > kFp8MaxHeads)
+        return fail(KVS_ERR_UNSUPPORTED, "fp8 chunks support at most %u kv heads", kFp8MaxHeads);
+    for (int32_t r = 0; r < nreq; ++r)
+        for (int32_t j = 0; j < reqs[r].num_chunks; ++j)
+            if ((uint64_t)reqs[r].chunks[j].base & 15)
+                return fail(KVS_ERR_UNSUPPORTED, "request %d chunk %d: fp8 chunks must be 16-byte aligned", r, j);
+    if (pl.addr_or & 15) return fail(KVS_ERR_UNSUPPORTED, "fp8 calls need 16-byte aligned planes");
+    if (flags & KVS_F_VALIDATE) {
+        rc = check_overlaps(g, cache, reqs, nreq, retrieve, true);
+        if (rc) return rc;
+    }
+    if (pl.num_device + pl.num_host == 0) return KVS_OK;
+    DevState* stp = nullptr;
+    rc = get_state(&stp);
+    if (rc) return rc;
+    DevState& st = *stp;
+    rc = fill_plan(st, g, cache, reqs, nreq, retrieve, flags & ~KVS_F_NO_DEDUP, pl);
+    if (rc) return rc;
+    if (pl.any_dedup) {
+        for (size_t k = 0; k < pl.demoted.size(); ++k)
+            if (pl.demoted[k] >= 0)
+                return fail(KVS_ERR_ALIAS, "fp8 retrieval: physical block %d is named by two requests", pl.demoted[k]);
+    }
+    pl.blocks_cmp.clear();
+    cudaStream_t s = (cudaStream_t)stream;
+    Uploaded u;
+    rc = upload(st, pl, s, u);
+    if (rc) return rc;
+    SlotGuard guard{u.slot, s};
+    const int cap = (int)KVS_F_GET_MAX_CTAS(flags);
+    const uint32_t hd = (uint32_t)(g->num_kv_heads * g->head_dim);
+    auto fjob = [&](uint32_t first, uint32_t count) {
+        Fp8Job f{};
+        f.job = make_job(st, g, cache, pl, u, first, count, retrieve ? MODE_RETRIEVE : MODE_STORE);
+        const uint64_t run_codes = (uint64_t)g->block_size * hd;
+        f.job.pieces_per_run = (uint32_t)((run_codes + kFp8PieceCodes - 1) / kFp8PieceCodes);
+        f.job.num_pieces = (uint64_t)count * f.job.num_planes * f.job.blocks_per_chunk * f.job.pieces_per_run;
+        f.heads = (uint32_t)g->num_kv_heads;
+        f.head_dim = (uint32_t)g->head_dim;
+        f.scale_bytes = (uint32_t)fp8_scale_bytes(g);
+        return f;
+    };
+    auto run = [&](const Fp8Job& f, int grid) -> int {
+        cudaError_t e = retrieve ? launch_fp8_retrieve(f, grid, s) : launch_fp8_store(f, grid, s);
+        if (e != cudaSuccess) return fail(KVS_ERR_CUDA, "fp8 kernel launch failed: %s", cudaGetErrorString(e));
+        ++g_launches;
+        return KVS_OK;
+    };
+    if (pl.num_host) {
+        const Fp8Job f = fjob(pl.num_device, pl.num_host);
+        if (f.job.num_pieces >= (1ull << 31)) return fail(KVS_ERR_INVALID_ARG, "call too large: split it");
+        // Retrieval: a CTA keeps up to 32 KiB of codes in flight, half a link-kernel
+        // CTA's bytes, so it takes twice the link kernel's grid.  Store-back: one CTA
+        // per (chunk, plane) over the whole GPU (its two passes are not pipelined
+        // across segments, so a capped grid would be latency-bound).
+        const int grid = cap ? cap : (retrieve ? 2 * st.hostlink_ctas : 0);
+        rc = run(f, grid);
+        if (rc) return rc;
+    }
+    if (pl.num_device) {
+        const Fp8Job f = fjob(0, pl.num_device);
+        if (f.job.num_pieces >= (1ull << 31)) return fail(KVS_ERR_INVALID_ARG, "call too large: split it");
+        rc = run(f, cap);
+        if (rc) return rc;
+    }
+    if (flags & KVS_F_VALIDATE) {
+        KVS_CUDA(cudaEventRecord(u.slot->done, s));
         u.slot->used = true;
         guard.slot = nullptr;
         return read_error_word(st, s);
@@ -895,8 +1055,10 @@ int query_bw(DevState& st, kvs_bw_report* out, cudaStream_t s, int64_t probe_byt
     };
     if ((rc = probe_call(&rh, true, KVS_F_FORCE_HOSTLINK, &rep.retrieve_gbs[0])) ||
         (rc = probe_call(&rh, true, KVS_F_FORCE_HBMCOPY, &rep.retrieve_gbs[1])) ||
+        (rc = probe_call(&rh, true, KVS_F_FORCE_DMA, &rep.retrieve_dma_gbs)) ||
         (rc = probe_call(&rh, false, KVS_F_FORCE_HOSTLINK, &rep.store_gbs[0])) ||
         (rc = probe_call(&rh, false, KVS_F_FORCE_HBMCOPY, &rep.store_gbs[1])) ||
+        (rc = probe_call(&rh, false, KVS_F_FORCE_DMA, &rep.store_dma_gbs)) ||
         (rc = probe_call(&rd, true, KVS_F_FORCE_LDG, &rep.device_kernel_gbs[0])) ||
         (rc = probe_call(&rd, true, KVS_F_FORCE_TMA, &rep.device_kernel_gbs[1]))) {
         cleanup();
@@ -936,16 +1098,79 @@ int query_bw(DevState& st, kvs_bw_report* out, cudaStream_t s, int64_t probe_byt
     // host memory is erratic on buffers of tens of GiB (13-210 GB/s on 40 GiB,
     // by box and allocation), where SM loads keep the link's rate, so the
     // copy-engine variant is taken only when it wins the probe clearly.
+    // The same holds for the DMA variant (the copy engine again).  kvs_tune
+    // measures the caller's own call instead.
     constexpr double kHbmcopyMargin = 1.05;
-    st.retrieve_host = rep.retrieve_gbs[1] > kHbmcopyMargin * rep.retrieve_gbs[0] ? KVS_VARIANT_HBMCOPY
-                                                                                 : KVS_VARIANT_HOSTLINK;
-    st.store_host = rep.store_gbs[1] > kHbmcopyMargin * rep.store_gbs[0] ? KVS_VARIANT_HBMCOPY
-                                                                       : KVS_VARIANT_HOSTLINK;
+    auto pick = [&](double hostlink, double hbmcopy, double dma) {
+        int v = KVS_VARIANT_HOSTLINK;
+        double best = hostlink;
+        if (hbmcopy > kHbmcopyMargin * hostlink && hbmcopy > best) { v = KVS_VARIANT_HBMCOPY; best = hbmcopy; }
+        if (dma > kHbmcopyMargin * hostlink && dma > best) v = KVS_VARIANT_DMA;
+        return v;
+    };
+    st.retrieve_host = pick(rep.retrieve_gbs[0], rep.retrieve_gbs[1], rep.retrieve_dma_gbs);
+    st.store_host = pick(rep.store_gbs[0], rep.store_gbs[1], rep.store_dma_gbs);
     st.kernel_device = rep.device_kernel_gbs[1] > rep.device_kernel_gbs[0] ? KVS_KERNEL_TMA : KVS_KERNEL_LDG;
     rep.chosen_retrieve_host = st.retrieve_host;
     rep.chosen_store_host = st.store_host;
     rep.chosen_kernel_device = st.kernel_device;
     st.report = rep;
+    if (out) *out = rep;
+    return KVS_OK;
+}
+
+int tune(DevState& st, const kvs_geometry* g, const kvs_paged_cache* cache, const kvs_request* reqs,
+         int32_t nreq, cudaStream_t s, uint32_t flags, int32_t direction, int32_t reps, kvs_tune_report* out) {
+    const uint32_t forced = KVS_F_FORCE_HOSTLINK | KVS_F_FORCE_HBMCOPY | KVS_F_FORCE_DMA | KVS_F_FORCE_LDG |
+                            KVS_F_FORCE_TMA | KVS_F_LAYER_LAUNCHES | KVS_F_LAYER_SIGNAL;
+    if (flags & forced) return fail(KVS_ERR_INVALID_ARG, "kvs_tune chooses the variant: no FORCE or layer flags");
+    if (direction != KVS_DIR_RETRIEVE && direction != KVS_DIR_STORE)
+        return fail(KVS_ERR_INVALID_ARG, "direction must be KVS_DIR_RETRIEVE or KVS_DIR_STORE");
+    if (reps < 1 || reps > 1000) return fail(KVS_ERR_INVALID_ARG, "reps must be in [1, 1000]");
+    const bool retrieve = direction == KVS_DIR_RETRIEVE;
+    Plan pl;
+    int rc = validate_call(g, cache, reqs, nreq, pl);
+    if (rc) return rc;
+    kvs_tune_report rep{};
+    rep.direction = direction;
+    int64_t host_bytes = 0;
+    for (int32_t r = 0; r < nreq; ++r)
+        for (int32_t j = 0; j < reqs[r].num_chunks; ++j)
+            if (reqs[r].chunks[j].residency == KVS_SRC_HOST_PINNED)
+                host_bytes += (int64_t)2 * g->num_layers * reqs[r].chunks[j].num_tokens * (int64_t)pl.row_bytes;
+    rep.host_bytes = host_bytes;
+    rep.chosen = retrieve ? st.retrieve_host : st.store_host;
+    if (host_bytes == 0) {
+        if (out) *out = rep;
+        return KVS_OK;
+    }
+    const uint32_t cap = flags & 0xFFFF0000u, base = flags & ~0xFFFF0000u;
+    const bool dma_ok = dma_pitch(st, pl, (uint64_t)g->block_size * pl.row_bytes) != 0;
+    const uint32_t cand[3] = {KVS_F_FORCE_HOSTLINK | cap, KVS_F_FORCE_HBMCOPY, KVS_F_FORCE_DMA};
+    for (int v = 0; v < 3; ++v) {
+        if (v == 2 && !dma_ok) continue;
+        rc = copy_call(g, cache, reqs, nreq, (void*)s, base | cand[v], retrieve);   // untimed (validated if asked)
+        if (rc) return rc;
+        double best = 0;
+        rc = time_best(s, reps, &best, [&]() -> int {
+            return copy_call(g, cache, reqs, nreq, (void*)s, (base & ~KVS_F_VALIDATE) | cand[v], retrieve);
+        });
+        if (rc) return rc;
+        rep.gbs[v] = (double)host_bytes / (best * 1e6);
+    }
+    KVS_CUDA(cudaStreamSynchronize(s));
+    int v = 0;
+    for (int k = 1; k < 3; ++k)
+        if (rep.gbs[k] > rep.gbs[v]) v = k;
+    const int chosen = v == 0 ? KVS_VARIANT_HOSTLINK : v == 1 ? KVS_VARIANT_HBMCOPY : KVS_VARIANT_DMA;
+    if (retrieve) {
+        st.retrieve_host = chosen;
+        if (chosen == KVS_VARIANT_HOSTLINK && cap) st.hostlink_ctas = (int)KVS_F_GET_MAX_CTAS(flags);
+    } else {
+        st.store_host = chosen;
+        if (chosen == KVS_VARIANT_HOSTLINK && cap) st.store_ctas = (int)KVS_F_GET_MAX_CTAS(flags);
+    }
+    rep.chosen = chosen;
     if (out) *out = rep;
     return KVS_OK;
 }
@@ -991,6 +1216,20 @@ int kvs_store(const kvs_geometry* geom, const kvs_paged_cache* cache, const kvs_
     return copy_call(geom, cache, requests, num_requests, cuda_stream, flags, false);
 }
 
+int kvs_retrieve_fp8(const kvs_geometry* geom, const kvs_paged_cache* cache, const kvs_request* requests,
+                     int32_t num_requests, void* cuda_stream, uint32_t flags) {
+    std::lock_guard<std::mutex> lk(g_mu);
+    t_error.clear();
+    return fp8_call(geom, cache, requests, num_requests, cuda_stream, flags, true);
+}
+
+int kvs_store_fp8(const kvs_geometry* geom, const kvs_paged_cache* cache, const kvs_request* requests,
+                  int32_t num_requests, void* cuda_stream, uint32_t flags) {
+    std::lock_guard<std::mutex> lk(g_mu);
+    t_error.clear();
+    return fp8_call(geom, cache, requests, num_requests, cuda_stream, flags, false);
+}
+
 int kvs_retrieve_layers(const kvs_geometry* geom, const kvs_paged_cache* cache, const kvs_request* requests,
                         int32_t num_requests, int32_t layers_per_step, void* const* layer_events,
                         void* cuda_stream, uint32_t flags) {
@@ -1017,6 +1256,23 @@ int kvs_query_bw(kvs_bw_report* out, void* cuda_stream, int64_t probe_bytes) {
     int rc = get_state(&st);
     if (rc) return rc;
     return query_bw(*st, out, (cudaStream_t)cuda_stream, probe_bytes);
+}
+
+int kvs_tune(const kvs_geometry* geom, const kvs_paged_cache* cache, const kvs_request* requests,
+             int32_t num_requests, void* cuda_stream, uint32_t flags, int32_t direction, int32_t reps,
+             kvs_tune_report* out) {
+    std::lock_guard<std::mutex> lk(g_mu);
+    t_error.clear();
+    if (direction != KVS_DIR_RETRIEVE && direction != KVS_DIR_STORE)
+        return fail(KVS_ERR_INVALID_ARG, "direction must be KVS_DIR_RETRIEVE or KVS_DIR_STORE");
+    if (reps < 1 || reps > 1000) return fail(KVS_ERR_INVALID_ARG, "reps must be in [1, 1000]");
+    Plan pl;
+    int rc = validate_call(geom, cache, requests, num_requests, pl);      // before any device state
+    if (rc) return rc;
+    DevState* st = nullptr;
+    rc = get_state(&st);
+    if (rc) return rc;
+    return tune(*st, geom, cache, requests, num_requests, (cudaStream_t)cuda_stream, flags, direction, reps, out);
 }
 
 int kvs_get_choice(kvs_bw_report* out) {

@@ -1,0 +1,373 @@
+// kvs_fp8.cu -- retrieval from, and store-back into, fp8 chunks on sm_103a.
+//
+// A compressed fast-tier format (the paper keeps BF16 KV, Sec. 5 setup): a
+// chunk holds E4M3 codes of the OCP 8-bit floating point specification
+// (revision 1.0) and one binary32 scale per (layer, K/V, head), so a
+// retrieval moves half the bytes of a BF16 chunk over the host link:
+//
+//   chunk  [scales: 2L*H binary32 at (2l+kv)*H + h, padded to scale_bytes]
+//          [codes:  [L][2][n][H][D] E4M3 bytes]
+//   plane  BF16 [NB][B][H][D] per (layer, K/V)
+//
+//   retrieve  plane = bf16_rn(fp32(code) *rn scale); a NaN product gives 0x7FFF
+//   store     per (chunk, layer, K/V, head): amax over the finite elements,
+//             scale = amax /rn 448 (1 when amax is 0), code = e4m3 of
+//             x /rn scale, rounded to nearest even and saturated at +-448;
+//             NaN gives the code 0x7F
+//
+// Every element conversion uses the hardware conversions of sm_89+ (E4M3 <->
+// f16 pairs, f32 -> bf16 pairs) and IEEE round-to-nearest multiply / divide;
+// NaN results and magnitudes at or below 2^-10 (which round to zero) are set
+// explicitly, so the result does not depend on how a conversion treats NaN
+// signs or binary32 subnormals.
+//
+// Retrieval is bound by the host link (or HBM for device chunks): a persistent
+// grid of 128-thread CTAs walks 16 KiB pieces of codes; each thread keeps two
+// pieces' worth of 16-byte code vectors in registers, so the next piece's
+// loads are in flight while the current one is converted and stored.  The H
+// scales of a piece's plane are loaded once per piece by H threads (one 4-byte
+// load each, beside the codes) and shared through shared memory, instead of
+// one scale load per vector.  Store-back runs one 256-thread CTA per (chunk,
+// plane) over the whole GPU: a first pass takes the per-head amax, a second
+// quantises (the re-read hits L2 or HBM; the destination write over the host
+// link is the bound); both passes keep four vectors per thread in flight.
+#include <cuda_bf16.h>
+#include <cuda_fp16.h>
+#include <cuda_fp8.h>
+
+#include <algorithm>
+#include <cstdint>
+
+#include "kvs.h"
+#include "kvs_internal.h"
+
+namespace kvs {
+namespace {
+
+constexpr int kRtThreads = 128;
+constexpr int kRtVec = 8;                            // 16-code vectors per thread per piece
+static_assert(kRtThreads * kRtVec * 16 == kFp8PieceCodes, "a piece is one vector set per CTA");
+constexpr int kStThreads = 256;
+
+struct Fp8Piece {
+    uint64_t codes;      // first code of the piece
+    uint64_t out;        // first BF16 element of the piece in the plane
+    uint64_t scales;     // scale block row of the piece's plane: H binary32
+    uint32_t len;        // codes in the piece (a multiple of 16)
+    uint32_t vec0;       // index of the piece's first vector within its run
+};
+
+// Piece q -> addresses; false for pieces with nothing to move.  Runs are
+// (entry, plane, block) as for BF16 copies; a run holds ntok rows of H*D codes.
+__device__ __forceinline__ bool fp8_piece(const Fp8Job& f, uint32_t q, Fp8Piece& pc) {
+    const Job& j = f.job;
+    const uint32_t hd = f.heads * f.head_dim;
+    const uint32_t run = q / j.pieces_per_run;
+    const uint32_t k = q - run * j.pieces_per_run;
+    const uint32_t per_entry = j.num_planes * j.blocks_per_chunk;
+    const uint32_t e = run / per_entry;
+    const uint32_t rem = run - e * per_entry;
+    const uint32_t pr = rem / j.blocks_per_chunk;
+    const uint32_t i = rem - pr * j.blocks_per_chunk;
+    const uint32_t p = j.plane_begin + pr;
+    const int32_t blk = __ldg(j.blocks + (size_t)(j.entry_base + e) * j.blocks_per_chunk + i);
+    const Entry en = j.entries[e];
+    const int64_t first = (int64_t)i * j.block_size;
+    const int64_t ntok = min((int64_t)j.block_size, (int64_t)en.n_tok - first);
+    if (ntok <= 0 || blk < 0) return false;
+    if (blk >= j.num_blocks) {
+        atomicCAS(j.err, 0, KVS_ERR_BOUNDS);
+        return false;
+    }
+    const uint64_t run_codes = (uint64_t)ntok * hd;
+    const uint64_t off = (uint64_t)k * kFp8PieceCodes;
+    if (off >= run_codes) return false;
+    pc.len = (uint32_t)min((uint64_t)kFp8PieceCodes, run_codes - off);
+    pc.vec0 = (uint32_t)(off / 16);
+    pc.codes = en.chunk + f.scale_bytes + ((uint64_t)p * (uint64_t)en.n_tok + (uint64_t)first) * hd + off;
+    pc.out = j.planes[p] + ((uint64_t)blk * j.block_size) * hd * 2 + off * 2;
+    pc.scales = en.chunk + (uint64_t)p * f.heads * 4;
+    return true;
+}
+
+__device__ __forceinline__ uint4 ld_nc16(uint64_t a) {
+    uint4 r;
+    asm volatile("ld.global.nc.L1::no_allocate.v4.u32 {%0,%1,%2,%3}, [%4];"
+                 : "=r"(r.x), "=r"(r.y), "=r"(r.z), "=r"(r.w) : "l"(a));
+    return r;
+}
+
+__device__ __forceinline__ void st_cs16(uint64_t a, const uint4& v) {
+    asm volatile("st.global.cs.v4.u32 [%0], {%1,%2,%3,%4};"
+                 :: "l"(a), "r"(v.x), "r"(v.y), "r"(v.z), "r"(v.w) : "memory");
+}
+
+// Two E4M3 codes (low byte first) times `s` -> two BF16 (low half first).
+__device__ __forceinline__ uint32_t e4m3x2_to_bf16x2(uint32_t two, float s) {
+    const __half2_raw hr = __nv_cvt_fp8x2_to_halfraw2((__nv_fp8x2_storage_t)(two & 0xFFFFu), __NV_E4M3);
+    __half2 h;
+    *reinterpret_cast<__half2_raw*>(&h) = hr;
+    const float2 v = __half22float2(h);                          // exact
+    const float a = __fmul_rn(v.x, s), b = __fmul_rn(v.y, s);
+    const __nv_bfloat162 r = __floats2bfloat162_rn(a, b);
+    uint32_t bits = *reinterpret_cast<const uint32_t*>(&r);
+    if (a != a) bits = (bits & 0xFFFF0000u) | 0x00007FFFu;
+    if (b != b) bits = (bits & 0x0000FFFFu) | 0x7FFF0000u;
+    return bits;
+}
+
+// 16 codes -> 32 bytes of BF16.
+__device__ __forceinline__ void dequant16(const uint4& c, float s, uint4& lo, uint4& hi) {
+    lo.x = e4m3x2_to_bf16x2(c.x, s);
+    lo.y = e4m3x2_to_bf16x2(c.x >> 16, s);
+    lo.z = e4m3x2_to_bf16x2(c.y, s);
+    lo.w = e4m3x2_to_bf16x2(c.y >> 16, s);
+    hi.x = e4m3x2_to_bf16x2(c.z, s);
+    hi.y = e4m3x2_to_bf16x2(c.z >> 16, s);
+    hi.z = e4m3x2_to_bf16x2(c.w, s);
+    hi.w = e4m3x2_to_bf16x2(c.w >> 16, s);
+}
+
+// A piece's codes in registers; thread t < H also holds the scale of head t,
+// loaded once per piece (not once per vector) beside the codes.
+struct RtRegs {
+    uint4 c[kRtVec];
+    float s;
+};
+
+__device__ __forceinline__ void rt_load(const Fp8Job& f, const Fp8Piece& pc, RtRegs& r) {
+    const uint32_t nv = pc.len / 16;
+#pragma unroll
+    for (int u = 0; u < kRtVec; ++u) {
+        const uint32_t v = threadIdx.x + u * kRtThreads;
+        if (v < nv) r.c[u] = ld_nc16(pc.codes + (uint64_t)v * 16);
+    }
+    if (threadIdx.x < f.heads) r.s = __ldg(reinterpret_cast<const float*>(pc.scales) + threadIdx.x);
+}
+
+// Publishes the piece's scales in shared memory (after every thread has finished
+// with the previous piece's), then converts and stores this thread's vectors.
+__device__ __forceinline__ void rt_store(const Fp8Job& f, const Fp8Piece& pc, const RtRegs& r, float* sm_scale) {
+    const uint32_t vph = f.head_dim / 16, vpr = f.heads * vph;
+    const uint32_t nv = pc.len / 16;
+    __syncthreads();
+    if (threadIdx.x < f.heads) sm_scale[threadIdx.x] = r.s;
+    __syncthreads();
+#pragma unroll
+    for (int u = 0; u < kRtVec; ++u) {
+        const uint32_t v = threadIdx.x + u * kRtThreads;
+        if (v < nv) {
+            uint4 lo, hi;
+            dequant16(r.c[u], sm_scale[((pc.vec0 + v) % vpr) / vph], lo, hi);
+            st_cs16(pc.out + (uint64_t)v * 32, lo);
+            st_cs16(pc.out + (uint64_t)v * 32 + 16, hi);
+        }
+    }
+}
+
+__device__ __forceinline__ bool rt_next(const Fp8Job& f, uint32_t n, uint32_t& q, Fp8Piece& pc) {
+    while (q < n) {
+        const uint32_t cur = q;
+        q += gridDim.x;
+        if (fp8_piece(f, cur, pc)) return true;
+    }
+    return false;
+}
+
+// Every thread of a CTA walks the same sequence of pieces (the piece index
+// depends only on blockIdx), so the barriers in rt_store are reached by all.
+__global__ void __launch_bounds__(kRtThreads) kvs_fp8_retrieve_kernel(const Fp8Job f, uint32_t num_pieces) {
+    __shared__ float sm_scale[kFp8MaxHeads];
+    RtRegs ra, rb;
+    Fp8Piece pa, pb;
+    uint32_t q = blockIdx.x;
+    bool ha = rt_next(f, num_pieces, q, pa);
+    if (ha) rt_load(f, pa, ra);
+    while (ha) {
+        const bool hb = rt_next(f, num_pieces, q, pb);
+        if (hb) rt_load(f, pb, rb);
+        rt_store(f, pa, ra, sm_scale);
+        if (!hb) break;
+        ha = rt_next(f, num_pieces, q, pa);
+        if (ha) rt_load(f, pa, ra);
+        rt_store(f, pb, rb, sm_scale);
+    }
+}
+
+// ---------------------------------------------------------------------------
+// Store-back (quantise)
+// ---------------------------------------------------------------------------
+
+// Largest |x| bit pattern among the finite BF16 values of a 16-byte vector
+// (|x| of a finite BF16 orders like its bits with the sign cleared).
+__device__ __forceinline__ uint32_t amax_bits8(const uint4& v) {
+    uint32_t m = 0;
+    const uint32_t w[4] = {v.x, v.y, v.z, v.w};
+#pragma unroll
+    for (int k = 0; k < 4; ++k) {
+        const uint32_t a = w[k] & 0x7FFFu, b = (w[k] >> 16) & 0x7FFFu;
+        if (a < 0x7F80u) m = max(m, a);
+        if (b < 0x7F80u) m = max(m, b);
+    }
+    return m;
+}
+
+__device__ __forceinline__ float bf16_lo(uint32_t w) { return __uint_as_float(w << 16); }
+__device__ __forceinline__ float bf16_hi(uint32_t w) { return __uint_as_float(w & 0xFFFF0000u); }
+
+// One E4M3 code of q: NaN -> 0x7F; |q| <= 2^-10 rounds to a signed zero; the
+// rest through the saturating round-to-nearest-even conversion.
+__device__ __forceinline__ uint32_t fix_code(float q, uint32_t hw) {
+    if (q != q) return 0x7Fu;
+    if (fabsf(q) <= 0x1p-10f) return (__float_as_uint(q) >> 24) & 0x80u;
+    return hw;
+}
+
+__device__ __forceinline__ uint32_t e4m3x2(float a, float b) {
+    const uint32_t hw = (uint32_t)__nv_cvt_float2_to_fp8x2(make_float2(a, b), __NV_SATFINITE, __NV_E4M3);
+    return fix_code(a, hw & 0xFFu) | (fix_code(b, hw >> 8) << 8);
+}
+
+// 16 BF16 (two vectors) divided by `s` -> 16 codes.
+__device__ __forceinline__ uint4 quant16(const uint4& a, const uint4& b, float s) {
+    const uint32_t w[8] = {a.x, a.y, a.z, a.w, b.x, b.y, b.z, b.w};
+    uint32_t c[8];
+#pragma unroll
+    for (int k = 0; k < 8; ++k)
+        c[k] = e4m3x2(__fdiv_rn(bf16_lo(w[k]), s), __fdiv_rn(bf16_hi(w[k]), s));
+    return make_uint4(c[0] | (c[1] << 16), c[2] | (c[3] << 16), c[4] | (c[5] << 16), c[6] | (c[7] << 16));
+}
+
+constexpr int kStUnroll = 4;                         // vectors per thread in flight per step
+
+// One CTA per (entry, plane) segment: the chunk's n tokens of that plane.
+__global__ void __launch_bounds__(kStThreads) kvs_fp8_store_kernel(const Fp8Job f, uint32_t num_segments) {
+    __shared__ uint32_t amax[kFp8MaxHeads];
+    __shared__ float scale[kFp8MaxHeads];
+    const Job& j = f.job;
+    const uint32_t H = f.heads, vph = f.head_dim / 16, vpr = H * vph;
+    const uint64_t row2 = (uint64_t)H * f.head_dim * 2;          // BF16 bytes per token row
+    for (uint32_t seg = blockIdx.x; seg < num_segments; seg += gridDim.x) {
+        const uint32_t e = seg / j.num_planes;
+        const uint32_t p = j.plane_begin + (seg - e * j.num_planes);
+        const Entry en = j.entries[e];
+        const uint32_t n = (uint32_t)en.n_tok;
+        const int32_t* blocks = j.blocks + (size_t)(j.entry_base + e) * j.blocks_per_chunk;
+        const uint64_t plane = j.planes[p];
+        const uint64_t codes = en.chunk + f.scale_bytes + (uint64_t)p * n * vpr * 16;
+        const uint32_t nvec = n * vpr;
+        // source address of vector v (16 BF16 = 32 bytes), or 0 for a bad block
+        auto src_of = [&](uint32_t v, uint32_t& h) -> uint64_t {
+            const uint32_t i = v / vpr, w = v - i * vpr;
+            h = w / vph;
+            const int32_t blk = __ldg(blocks + i / j.block_size);
+            if (blk < 0 || blk >= j.num_blocks) return 0;
+            return plane + ((uint64_t)blk * j.block_size + i % j.block_size) * row2 + (uint64_t)w * 32;
+        };
+        for (uint32_t h = threadIdx.x; h < H; h += blockDim.x) amax[h] = 0;
+        __syncthreads();
+        // pass 1: per-head amax over the finite elements of this chunk's plane p
+        uint32_t cur_h = 0xFFFFFFFFu, m = 0;
+        bool bad = false;
+        for (uint32_t v0 = threadIdx.x; v0 < nvec; v0 += blockDim.x * kStUnroll) {
+            uint4 a[kStUnroll], b[kStUnroll];
+            uint32_t hh[kStUnroll];
+            bool ok[kStUnroll];
+#pragma unroll
+            for (int u = 0; u < kStUnroll; ++u) {
+                const uint32_t v = v0 + u * blockDim.x;
+                ok[u] = false;
+                if (v < nvec) {
+                    const uint64_t src = src_of(v, hh[u]);
+                    if (src) {
+                        a[u] = ld_nc16(src);
+                        b[u] = ld_nc16(src + 16);
+                        ok[u] = true;
+                    } else {
+                        bad = true;
+                    }
+                }
+            }
+#pragma unroll
+            for (int u = 0; u < kStUnroll; ++u) {
+                if (!ok[u]) continue;
+                const uint32_t lm = max(amax_bits8(a[u]), amax_bits8(b[u]));
+                if (hh[u] != cur_h) {
+                    if (cur_h != 0xFFFFFFFFu) atomicMax(&amax[cur_h], m);
+                    cur_h = hh[u];
+                    m = 0;
+                }
+                m = max(m, lm);
+            }
+        }
+        if (cur_h != 0xFFFFFFFFu) atomicMax(&amax[cur_h], m);
+        if (bad) atomicCAS(j.err, 0, KVS_ERR_BOUNDS);
+        __syncthreads();
+        for (uint32_t h = threadIdx.x; h < H; h += blockDim.x) {
+            const float a = __uint_as_float(amax[h] << 16);
+            const float s = a > 0.0f ? __fdiv_rn(a, 448.0f) : 1.0f;
+            scale[h] = s;
+            *reinterpret_cast<float*>(en.chunk + ((uint64_t)p * H + h) * 4) = s;
+        }
+        __syncthreads();
+        // pass 2: quantise
+        for (uint32_t v0 = threadIdx.x; v0 < nvec; v0 += blockDim.x * kStUnroll) {
+            uint4 a[kStUnroll], b[kStUnroll];
+            uint32_t hh[kStUnroll];
+            bool ok[kStUnroll];
+#pragma unroll
+            for (int u = 0; u < kStUnroll; ++u) {
+                const uint32_t v = v0 + u * blockDim.x;
+                ok[u] = false;
+                if (v < nvec) {
+                    const uint64_t src = src_of(v, hh[u]);
+                    if (src) {
+                        a[u] = ld_nc16(src);
+                        b[u] = ld_nc16(src + 16);
+                        ok[u] = true;
+                    }
+                }
+            }
+#pragma unroll
+            for (int u = 0; u < kStUnroll; ++u)
+                if (ok[u]) st_cs16(codes + (uint64_t)(v0 + u * blockDim.x) * 16, quant16(a[u], b[u], scale[hh[u]]));
+        }
+        __syncthreads();                                   // amax / scale are reused by the next segment
+    }
+}
+
+int g_sms = 0;
+
+int sm_count() {
+    if (g_sms == 0) {
+        int dev = 0, n = 0;
+        cudaGetDevice(&dev);
+        cudaDeviceGetAttribute(&n, cudaDevAttrMultiProcessorCount, dev);
+        g_sms = n > 0 ? n : 1;
+    }
+    return g_sms;
+}
+
+}  // namespace
+
+cudaError_t launch_fp8_retrieve(const Fp8Job& fj, int grid, cudaStream_t s) {
+    const uint64_t n = fj.job.num_pieces;
+    if (n == 0) return cudaSuccess;
+    int per_sm = 0;
+    cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, kvs_fp8_retrieve_kernel, kRtThreads, 0);
+    const int full = sm_count() * std::max(per_sm, 1);
+    if (grid <= 0 || grid > full) grid = full;
+    if ((uint64_t)grid > n) grid = (int)n;
+    kvs_fp8_retrieve_kernel<<<grid, kRtThreads, 0, s>>>(fj, (uint32_t)n);
+    return cudaGetLastError();
+}
+
+cudaError_t launch_fp8_store(const Fp8Job& fj, int grid, cudaStream_t s) {
+    const uint64_t segs = (uint64_t)fj.job.num_entries * fj.job.num_planes;
+    if (segs == 0) return cudaSuccess;
+    if (grid <= 0 || (uint64_t)grid > segs) grid = (int)segs;
+    kvs_fp8_store_kernel<<<grid, kStThreads, 0, s>>>(fj, (uint32_t)segs);
+    return cudaGetLastError();
+}
+
+}  // namespace kvs

@@ -72,6 +72,24 @@ struct Signal {
 };
 cudaError_t launch_link_signal(const Job& job, const Signal& sig, int grid, cudaStream_t s);
 
+// fp8 chunks: [scales: 2L*H binary32, zero-padded to scale_bytes][codes [L][2][n][H][D] E4M3].
+// The Job's planes are BF16 ([NB][B][H][D], row_bytes = 2*H*D); entries point at chunk
+// buffers (scale block first); blocks_per_chunk / block_size / planes as for BF16 copies.
+struct Fp8Job {
+    Job      job;                // mode MODE_RETRIEVE (dequantise) or MODE_STORE (quantise)
+    uint32_t heads;              // H
+    uint32_t head_dim;           // D, a multiple of 16
+    uint32_t scale_bytes;        // bytes of the scale block, a multiple of 256
+};
+constexpr uint32_t kFp8MaxHeads = 128;
+// Retrieval: a persistent grid of `grid` CTAs (<= 0: fill the GPU) over pieces of at
+// most 16 KiB of codes, double-buffered; the number of pieces is in job.num_pieces.
+cudaError_t launch_fp8_retrieve(const Fp8Job& fj, int grid, cudaStream_t s);
+// Store-back: one CTA per (entry, plane), or a grid-stride loop over them with `grid` > 0.
+cudaError_t launch_fp8_store(const Fp8Job& fj, int grid, cudaStream_t s);
+// Codes per retrieval piece (16 KiB).
+constexpr uint32_t kFp8PieceCodes = 16384;
+
 // One CTA waits (bounded by limit_ns) on an mbarrier phase that nothing
 // completes, then records KVS_ERR_TIMEOUT: exercises the bounded-wait path.
 cudaError_t launch_stall(int32_t* err, uint64_t limit_ns, cudaStream_t s);

@@ -44,6 +44,9 @@ KVS_F_FORCE_TMA = 1 << 4
 KVS_F_NO_DEDUP = 1 << 5
 KVS_F_LAYER_LAUNCHES = 1 << 6
 KVS_F_LAYER_SIGNAL = 1 << 7
+KVS_F_FORCE_DMA = 1 << 8
+KVS_DIR_RETRIEVE = 0
+KVS_DIR_STORE = 1
 
 
 def KVS_F_MAX_CTAS(n: int) -> int:
@@ -52,6 +55,8 @@ def KVS_F_MAX_CTAS(n: int) -> int:
 
 KVS_VARIANT_HOSTLINK = 1
 KVS_VARIANT_HBMCOPY = 2
+KVS_VARIANT_DMA = 3
+VARIANT_NAMES = {1: "hostlink", 2: "hbmcopy", 3: "dma"}
 KVS_KERNEL_LDG = 1
 KVS_KERNEL_TMA = 2
 
@@ -59,6 +64,7 @@ EXPORTED = ("kvs_retrieve", "kvs_store", "kvs_query_bw", "kvs_get_choice", "kvs_
             "kvs_enqueue_error_read",
             "kvs_last_error", "kvs_shutdown", "kvs_version", "kvs_selftest_wait_timeout",
             "kvs_stat_launches", "kvs_retrieve_noalloc", "kvs_retrieve_layers", "kvs_store_layers",
+            "kvs_retrieve_fp8", "kvs_store_fp8", "kvs_tune",
             "kvs_tier_create", "kvs_tier_destroy", "kvs_tier_commit", "kvs_tier_staged",
             "kvs_tier_begin_retrieval", "kvs_tier_end_retrieval", "kvs_tier_cancel", "kvs_tier_ordinary",
             "kvs_tier_claim_state", "kvs_tier_object", "kvs_tier_stats_get", "kvs_tier_slot")
@@ -67,6 +73,10 @@ KVS_CLAIM_TRANSFERRING, KVS_CLAIM_RELEASED, KVS_CLAIM_CANCELLED, KVS_CLAIM_ORDIN
 CLAIM_NAMES = {0: "None", 1: "Planned", 2: "Staging", 3: "StageReady", 4: "Transferring",
                5: "Released", 6: "Cancelled", 7: "Ordinary"}
 KVS_NOALLOC_SCRATCH_BYTES = 1 << 20
+
+
+def KVS_FP8_SCALE_BYTES(L: int, H: int) -> int:
+    return (2 * L * H * 4 + 255) // 256 * 256
 
 
 class KvsError(RuntimeError):
@@ -104,7 +114,8 @@ class kvs_bw_report(ctypes.Structure):
                 ("chosen_retrieve_host", ctypes.c_int32), ("chosen_store_host", ctypes.c_int32),
                 ("chosen_kernel_device", ctypes.c_int32), ("num_sms", ctypes.c_int32),
                 ("hostlink_ctas", ctypes.c_int32), ("store_ctas", ctypes.c_int32),
-                ("probe_bytes", ctypes.c_int64)]
+                ("probe_bytes", ctypes.c_int64), ("retrieve_dma_gbs", ctypes.c_double),
+                ("store_dma_gbs", ctypes.c_double)]
 
     def as_dict(self) -> dict:
         out = {}
@@ -112,6 +123,11 @@ class kvs_bw_report(ctypes.Structure):
             v = getattr(self, name)
             out[name] = list(v) if isinstance(v, ctypes.Array) else v
         return out
+
+
+class kvs_tune_report(ctypes.Structure):
+    _fields_ = [("gbs", ctypes.c_double * 3), ("host_bytes", ctypes.c_int64), ("chosen", ctypes.c_int32),
+                ("direction", ctypes.c_int32)]
 
 
 class kvs_tier_config(ctypes.Structure):
@@ -152,7 +168,7 @@ def lib():
                                   "`python -m paper_2609_35065_gb300.build`")
             L = ctypes.CDLL(path)
             P = ctypes.c_void_p
-            for name in ("kvs_retrieve", "kvs_store", "kvs_retrieve_noalloc"):
+            for name in ("kvs_retrieve", "kvs_store", "kvs_retrieve_noalloc", "kvs_retrieve_fp8", "kvs_store_fp8"):
                 fn = getattr(L, name)
                 fn.argtypes = [ctypes.POINTER(kvs_geometry), ctypes.POINTER(kvs_paged_cache),
                                ctypes.POINTER(kvs_request), ctypes.c_int32, P, ctypes.c_uint32]
@@ -187,6 +203,10 @@ def lib():
                 fn.restype = ctypes.c_int
             L.kvs_tier_slot.argtypes = [P, ctypes.c_int64]
             L.kvs_tier_slot.restype = ctypes.c_void_p
+            L.kvs_tune.argtypes = [ctypes.POINTER(kvs_geometry), ctypes.POINTER(kvs_paged_cache),
+                                   ctypes.POINTER(kvs_request), ctypes.c_int32, P, ctypes.c_uint32,
+                                   ctypes.c_int32, ctypes.c_int32, ctypes.POINTER(kvs_tune_report)]
+            L.kvs_tune.restype = ctypes.c_int
             L.kvs_query_bw.argtypes = [ctypes.POINTER(kvs_bw_report), P, ctypes.c_int64]
             L.kvs_query_bw.restype = ctypes.c_int
             L.kvs_get_choice.argtypes = [ctypes.POINTER(kvs_bw_report)]
@@ -386,6 +406,18 @@ def kvs_query_bw(stream=None, probe_bytes: int = 0) -> dict:
     return rep.as_dict()
 
 
+def kvs_tune(geom, planes, num_blocks, requests, stream=None, flags: int = 0,
+             direction: int = KVS_DIR_RETRIEVE, reps: int = 3) -> dict:
+    """Time this call under each host-chunk variant, adopt the fastest as the default for
+    its direction, and return {"gbs": [hostlink, hbmcopy, dma], "chosen": ..., ...}."""
+    g = _geometry(geom)
+    m = _Marshalled(planes, num_blocks, requests)
+    rep = kvs_tune_report()
+    _check(lib().kvs_tune(ctypes.byref(g), ctypes.byref(m.cache), m.reqs, m.n, _stream(stream),
+                          ctypes.c_uint32(flags), int(direction), int(reps), ctypes.byref(rep)))
+    return {"gbs": list(rep.gbs), "host_bytes": rep.host_bytes, "chosen": rep.chosen, "direction": rep.direction}
+
+
 def kvs_get_choice() -> dict:
     rep = kvs_bw_report()
     _check(lib().kvs_get_choice(ctypes.byref(rep)))
@@ -431,6 +463,23 @@ def kvs_retrieve_noalloc(geom, planes, num_blocks, requests, stream=None, flags:
     m = _Marshalled(planes, num_blocks, requests)
     return _check(lib().kvs_retrieve_noalloc(ctypes.byref(g), ctypes.byref(m.cache), m.reqs, m.n,
                                              _stream(stream), ctypes.c_uint32(flags)))
+
+
+def kvs_retrieve_fp8(geom, planes, num_blocks, requests, stream=None, flags: int = 0) -> int:
+    """Dequantising retrieval from fp8 chunks (E4M3 codes with per-head scales) into
+    BF16 planes; chunk buffers are [scales][codes], see kvs.h."""
+    g = _geometry(geom)
+    m = _Marshalled(planes, num_blocks, requests)
+    return _check(lib().kvs_retrieve_fp8(ctypes.byref(g), ctypes.byref(m.cache), m.reqs, m.n,
+                                         _stream(stream), ctypes.c_uint32(flags)))
+
+
+def kvs_store_fp8(geom, planes, num_blocks, requests, stream=None, flags: int = 0) -> int:
+    """Quantising store-back from BF16 planes into fp8 chunks (scales and codes written)."""
+    g = _geometry(geom)
+    m = _Marshalled(planes, num_blocks, requests)
+    return _check(lib().kvs_store_fp8(ctypes.byref(g), ctypes.byref(m.cache), m.reqs, m.n,
+                                      _stream(stream), ctypes.c_uint32(flags)))
 
 
 # ---- fast tier ------------------------------------------------------------

@@ -25,7 +25,7 @@ def test_library_exports_every_declared_function():
     for n in names:
         assert hasattr(lib, n), n
     assert set(names) == set(kvs.EXPORTED)
-    assert kvs.kvs_version() == 10600
+    assert kvs.kvs_version() == 10800
 
 
 def test_struct_layouts_match_header():
@@ -33,7 +33,8 @@ def test_struct_layouts_match_header():
     assert ctypes.sizeof(kvs.kvs_chunk) == 16
     assert ctypes.sizeof(kvs.kvs_request) == 40
     assert ctypes.sizeof(kvs.kvs_paged_cache) == 16
-    assert ctypes.sizeof(kvs.kvs_bw_report) == 5 * 8 + 6 * 8 + 6 * 4 + 8
+    assert ctypes.sizeof(kvs.kvs_bw_report) == 5 * 8 + 6 * 8 + 6 * 4 + 8 + 2 * 8
+    assert ctypes.sizeof(kvs.kvs_tune_report) == 3 * 8 + 8 + 2 * 4
 
 
 class _Arena:

@@ -1,0 +1,147 @@
+"""fp8 chunks (E4M3 codes of the OCP OFP8 specification, revision 1.0, with per-head
+binary32 scales) through the C ABI against the CPU oracle, element by element.
+
+Retrieval dequantises into BF16 planes; store-back quantises BF16 planes into fp8
+chunks.  Both sides run the same round-to-nearest-even definitions, so the
+comparison is exact: planes bit for bit, chunks byte for byte (scales and codes).
+"""
+import numpy as np
+import pytest
+import torch
+
+import gpu_check as gc
+from paper_2609_35065_gb300 import buffers, kvs, synth
+
+pytestmark = pytest.mark.gpu
+
+
+@pytest.fixture(scope="module", autouse=True)
+def _cuda():
+    if not torch.cuda.is_available():
+        pytest.skip("no CUDA device")
+    torch.cuda.set_device(0)
+    yield
+    torch.cuda.synchronize()
+
+
+def _retrieve(buf, flags=kvs.KVS_F_VALIDATE, stream=None):
+    w = buf.workload
+    kvs.kvs_retrieve_fp8(w.geom, buf.plane_ptrs, w.num_blocks, buf.requests, stream, flags)
+
+
+def _store(buf, flags=kvs.KVS_F_VALIDATE, stream=None):
+    w = buf.workload
+    kvs.kvs_store_fp8(w.geom, buf.plane_ptrs, w.num_blocks, buf.store_requests, stream, flags)
+
+
+@pytest.mark.parametrize("residency", ["host", "device"])
+def test_fp8_small_retrieve_and_store(residency):
+    """L2 H4 D64, two 256-token chunks: dequantise, then quantise the same tokens back."""
+    w = synth.custom(2, 4, 64, 16, 256, 128, [512], [512], residency=residency, store_tokens=[0])
+    w.requests[0].store_tokens = 512
+    w.requests[0].store_first = 0
+    buf = buffers.allocate_fp8(w, store=True, store_residency=residency)
+    _retrieve(buf)
+    torch.cuda.synchronize()
+    gc.check_retrieve_fp8(buf)
+    _store(buf)
+    torch.cuda.synchronize()
+    gc.check_store_fp8(buf)
+
+
+@pytest.mark.parametrize("seed", range(24))
+def test_fp8_random_small_geometries(seed):
+    w = gc.random_fp8_workload(seed)
+    flags = [kvs.KVS_F_VALIDATE, 0, kvs.KVS_F_VALIDATE | kvs.KVS_F_MAX_CTAS(1 + seed % 5)][seed % 3]
+    buf = buffers.allocate_fp8(w, store=True, store_residency="host" if seed % 2 else "device")
+    s = torch.cuda.Stream()
+    _retrieve(buf, flags, s)
+    s.synchronize()
+    gc.check_retrieve_fp8(buf)
+    _store(buf, flags, s)
+    s.synchronize()
+    assert kvs.kvs_check_errors(s) == kvs.KVS_OK
+    gc.check_store_fp8(buf)
+
+
+def _bf16(x):
+    return np.array(x, dtype=np.float32).view(np.uint32) >> 16
+
+
+def test_fp8_special_values():
+    """Retrieval: NaN codes, the largest codes, subnormal codes and signed zeros under
+    NaN, infinite, zero, subnormal and huge scales.  Store-back: planes holding NaN,
+    infinities, signed zeros, BF16 subnormals, values at exact midpoints between E4M3
+    codes (a head whose amax is 448 has scale 1), and magnitudes at and around 2^-10."""
+    w = synth.custom(2, 2, 32, 16, 32, 8, [64], [32], store_tokens=[32])
+    buf = buffers.allocate_fp8(w, store=True)
+    ch = buf.chunks[0][0]
+    # one scale per (plane, head): 4 planes x 2 heads
+    scales = np.array([np.nan, np.inf, 0.0, 1e-40, 3e38, 1.0, -2.0, 0.5], dtype=np.float32)
+    sb = kvs.KVS_FP8_SCALE_BYTES(2, 2)
+    ch[:8 * 4].copy_(torch.from_numpy(scales.view(np.uint8)))
+    codes = np.arange(256, dtype=np.uint8)
+    body = np.resize(codes, ch.numel() - sb)
+    ch[sb:].copy_(torch.from_numpy(body))
+    torch.cuda.synchronize()
+    _retrieve(buf)
+    torch.cuda.synchronize()
+    gc.check_retrieve_fp8(buf)
+    # store-back of planes with special BF16 values
+    rng = np.random.default_rng(3)
+    mids = np.array([1.0625, 1.1875, 0.0009765625, -0.0009765625, 0.0014648438, 2 ** -10 * 1.0078125,
+                     13.0, 15.0, 17.0, 19.0, 240.0, 272.0, 464.0, 0.01367, 1e-40, -1e-40], dtype=np.float32)
+    special = np.concatenate([_bf16(mids), [0x7FC0, 0xFFC0, 0x7F80, 0xFF80, 0x0000, 0x8000, 0x0001, 0x8001]])
+    small = special[special != _bf16([464.0])[0]]                     # nothing above 448 in head 0
+    for p in range(4):
+        plane = buf.planes[p].view(-1)
+        vals = rng.choice(special, size=plane.numel()).astype(np.uint16).reshape(-1, 2, 32)
+        vals[:, 0, :] = rng.choice(small, size=vals[:, 0, :].shape)
+        # head 0 of every plane has amax exactly 448 (scale 1): its midpoints are exact ties
+        vals[:, 0, 0] = 0x43E0                                        # bf16 448.0
+        plane.copy_(torch.from_numpy(vals.reshape(-1).view(np.int16)))
+    torch.cuda.synchronize()
+    _store(buf)
+    torch.cuda.synchronize()
+    gc.check_store_fp8(buf)
+
+
+def test_fp8_llama8b_host_batch_retrieve_and_store():
+    """The 8B batch (16 requests x 2048 matched tokens, 128 chunks of 256 tokens: 2 GiB of
+    codes + scale blocks in pinned host memory) dequantised into the 20,000-block cache,
+    then stored back into fresh pinned fp8 chunks; every plane and chunk against the oracle."""
+    w = synth.llama8b()
+    for r in w.requests:
+        r.store_tokens = r.matched_tokens
+        r.store_first = 0
+    buf = buffers.allocate_fp8(w, store=True)
+    assert buf.payload_bytes == 128 * (2048 + (16 << 20))
+    s = torch.cuda.Stream()
+    kvs.kvs_retrieve_fp8(w.geom, buf.plane_ptrs, w.num_blocks, buf.requests, s, 0)
+    s.synchronize()
+    assert kvs.kvs_check_errors(s) == kvs.KVS_OK
+    gc.check_retrieve_fp8(buf)
+    kvs.kvs_store_fp8(w.geom, buf.plane_ptrs, w.num_blocks, buf.store_requests, s, 0)
+    s.synchronize()
+    assert kvs.kvs_check_errors(s) == kvs.KVS_OK
+    gc.check_store_fp8(buf)
+
+
+def test_fp8_refusals():
+    w = synth.custom(1, 2, 32, 16, 32, 8, [64, 64], [32, 32])
+    buf = buffers.allocate_fp8(w)
+    g = w.geom
+    # a physical block named by two requests
+    reqs = [buf.requests[0], kvs.RequestArg(buf.requests[0].block_table, buf.requests[1].chunks)]
+    with pytest.raises(kvs.KvsError) as ei:
+        kvs.kvs_retrieve_fp8(g, buf.plane_ptrs, w.num_blocks, reqs, None, 0)
+    assert ei.value.code == kvs.KVS_ERR_ALIAS
+    # head_dim not a multiple of 16 (the planes are large enough for the smaller rows)
+    with pytest.raises(kvs.KvsError) as ei:
+        kvs.kvs_retrieve_fp8((1, 2, 24, 2, 16, 32), buf.plane_ptrs, w.num_blocks, buf.requests[:1], None, 0)
+    assert ei.value.code == kvs.KVS_ERR_UNSUPPORTED
+    with pytest.raises(kvs.KvsError) as ei:
+        kvs.kvs_retrieve_fp8(g, buf.plane_ptrs, w.num_blocks, buf.requests, None, kvs.KVS_F_FORCE_HBMCOPY)
+    assert ei.value.code == kvs.KVS_ERR_UNSUPPORTED
+    torch.cuda.synchronize()
+    assert torch.all(buf.planes == buf.planes.view(-1)[0])

@@ -18,6 +18,7 @@ VARIANTS = {
     "default": 0,
     "hostlink": kvs.KVS_F_FORCE_HOSTLINK,
     "hbmcopy": kvs.KVS_F_FORCE_HBMCOPY,
+    "dma": kvs.KVS_F_FORCE_DMA,
     "ldg": kvs.KVS_F_FORCE_LDG,
     "tma": kvs.KVS_F_FORCE_TMA,
     "hbmcopy_tma": kvs.KVS_F_FORCE_HBMCOPY | kvs.KVS_F_FORCE_TMA,
