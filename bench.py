@@ -616,6 +616,9 @@ def run_ours(args):
     return 0
 
 
+COPY_ENGINE_ONLY = -1          # overlap variant: plain copy-engine copy of the pinned buffer, no scatter
+
+
 def overlap_measure(w, bw, side, variants, sampler=None):
     """Retrieval of workload ``w`` on the ``side`` stream while the current stream runs a
     bf16 8192 x 8192 GEMM loop, for each (name, flags) of ``variants``, alone and beside the
@@ -703,9 +706,19 @@ def overlap_measure(w, bw, side, variants, sampler=None):
         done = [t for t in (g0.elapsed_time(e) for e in gev) if t <= window_ms]
         return (2 * 8192 ** 3 * len(done) / (done[-1] / 1e3) / 1e12) if done else float("nan")
 
+    scratch = {}
+
     def copy(reqs, flags):
         """One retrieval of ``reqs``; KVS_F_LAYER_LAUNCHES here means one launch per layer
-        (a layer-wise call without events), which hands SMs back between layers."""
+        (a layer-wise call without events), which hands SMs back between layers.  The
+        flags value COPY_ENGINE_ONLY instead copies the pass's pinned buffer into one HBM
+        buffer with a plain cudaMemcpyAsync: the copy engine's rate with no scatter."""
+        if flags == COPY_ENGINE_ONLY:
+            if "dst" not in scratch:
+                scratch["dst"] = torch.empty_like(pinned, device="cuda")
+            with torch.cuda.stream(side):
+                scratch["dst"].copy_(pinned, non_blocking=True)
+            return
         if flags & kvs.KVS_F_LAYER_LAUNCHES:
             kvs.kvs_retrieve_layers(g, ptrs, w.num_blocks, reqs, 1, None, side, flags)
         else:
@@ -754,6 +767,7 @@ def overlap_measure(w, bw, side, variants, sampler=None):
             "gemm": "bf16 8192x8192x8192 torch.matmul loop on the main stream",
             "gemm_tflops_short_burst": round(2 * 8192 ** 3 / (gemm_ms / 1e3) / 1e12, 1)}
     del planes, pinned, refill_src, a, b, c
+    scratch.clear()
     torch.cuda.empty_cache()
     return results, info
 
@@ -878,7 +892,10 @@ def default_line_legs(args, buf, bw, stream, sampler, flags):
     # retrieval beside a bf16 GEMM loop (70B shape, 25% buffer), default cap
     side = torch.cuda.Stream(priority=-1)
     w70 = synth.llama70b(buffer_frac=0.25)
-    results, info = overlap_measure(w70, bw, side, [("default", 0), ("dma", kvs.KVS_F_FORCE_DMA)], sampler)
+    results, info = overlap_measure(w70, bw, side, [
+        ("default", 0),
+        ("prefetch_l2_24ctas", kvs.KVS_F_PREFETCH_L2 | kvs.KVS_F_MAX_CTAS(24)),
+        ("copy_engine_only", COPY_ENGINE_ONLY)], sampler)
     legs["overlap"] = {"workload": describe(w70), **info, "hostlink_ctas": kvs.kvs_get_choice()["hostlink_ctas"],
                        "side_stream": "high priority", **results}
     return legs
@@ -949,6 +966,34 @@ def run_fp8(args):
                       "tokens_per_s": round(w.matched_tokens / sm, 1), "ms": round(sm * 1e3, 4),
                       "clocks": sampler.summary(t1, t2)},
             "host_link_peak_gbs": round(host_peak, 2), "d2h_link_peak_gbs": round(d2h_peak, 2)}
+    # the same chunks staged in HBM: retrieve reads the codes (half the BF16 bytes) and writes
+    # BF16 planes, store reads the planes and writes codes; 1.5 x the BF16 payload either way
+    if not args.no_extras:
+        hbm_peak = max(measured_peaks().get("hbm_gbs", HBM_FALLBACK_GBS), bw["hbm_copy_gbs"])
+        dev = {}
+        for name, pool in (("chunks", fb.pools[0]), ("store", fb.pools[-1])):
+            dev[name] = pool.to("cuda")
+        def dev_reqs(reqs, pool, dpool):
+            base = int(pool.data_ptr())
+            return [kvs.RequestArg(r.block_table, [kvs.ChunkArg(int(dpool.data_ptr()) + (kvs._addr(c.base) - base),
+                                                               c.num_tokens, kvs.KVS_SRC_DEVICE) for c in r.chunks],
+                                   r.first_token) for r in reqs]
+        dreq = dev_reqs(fb.requests, fb.pools[0], dev["chunks"])
+        dsto = dev_reqs(fb.store_requests, fb.pools[-1], dev["store"])
+        payload16 = w.matched_tokens * token_bytes(g)
+        kvs.kvs_retrieve_fp8(g, fb.plane_ptrs, w.num_blocks, dreq, stream, kvs.KVS_F_VALIDATE)
+        kvs.kvs_store_fp8(g, fb.plane_ptrs, w.num_blocks, dsto, stream, kvs.KVS_F_VALIDATE)
+        rd = statistics.mean(timed(lambda: kvs.kvs_retrieve_fp8(g, fb.plane_ptrs, w.num_blocks, dreq, stream, 0),
+                                   args.steps))
+        sd = statistics.mean(timed(lambda: kvs.kvs_store_fp8(g, fb.plane_ptrs, w.num_blocks, dsto, stream, 0),
+                                   args.steps))
+        line["hbm_source"] = {
+            "retrieve": {"gbs_rw": round(1.5 * payload16 / rd / 1e9, 1), "frac_of_hbm": round(1.5 * payload16 / rd / 1e9 / hbm_peak, 4),
+                         "tokens_per_s": round(w.matched_tokens / rd, 1), "ms": round(rd * 1e3, 4)},
+            "store": {"gbs_rw": round(1.5 * payload16 / sd / 1e9, 1), "frac_of_hbm": round(1.5 * payload16 / sd / 1e9 / hbm_peak, 4),
+                      "tokens_per_s": round(w.matched_tokens / sd, 1), "ms": round(sd * 1e3, 4)},
+            "bytes_counted": "1.5 x BF16 payload (codes read + BF16 written, or BF16 read + codes written)",
+            "hbm_peak_gbs": round(hbm_peak, 1)}
     print(json.dumps(line), flush=True)
     return 0
 
@@ -971,6 +1016,9 @@ def run_overlap(args):
                 ("hostlink_24ctas", kvs.KVS_F_FORCE_HOSTLINK | kvs.KVS_F_MAX_CTAS(24)),
                 ("hbmcopy", kvs.KVS_F_FORCE_HBMCOPY),
                 ("dma", kvs.KVS_F_FORCE_DMA),
+                ("prefetch_l2_12ctas", kvs.KVS_F_PREFETCH_L2 | kvs.KVS_F_MAX_CTAS(12)),
+                ("prefetch_l2_24ctas", kvs.KVS_F_PREFETCH_L2 | kvs.KVS_F_MAX_CTAS(24)),
+                ("copy_engine_only", COPY_ENGINE_ONLY),
                 ("layer_launches", kvs.KVS_F_LAYER_LAUNCHES),
                 ("layer_launches_96ctas", kvs.KVS_F_LAYER_LAUNCHES | kvs.KVS_F_MAX_CTAS(96))]
     sampler = ClockSampler(torch.cuda.current_device())

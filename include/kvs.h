@@ -96,6 +96,11 @@ extern "C" {
                                           them.  Needs equally spaced planes (plane p at
                                           plane 0 + p * pitch, as in one [2L][...] cache
                                           allocation); KVS_ERR_UNSUPPORTED otherwise      */
+#define KVS_F_PREFETCH_L2    (1u << 9) /* retrieval of host chunks on the host-link kernel:
+                                          each CTA keeps its upcoming pieces in flight as
+                                          bulk L2 prefetches, so the bytes in flight wait
+                                          in L2 rather than in registers and a small
+                                          KVS_F_MAX_CTAS grid can hold the link rate      */
 #define KVS_F_MAX_CTAS(n)    ((((uint32_t)(n)) & 0xFFFFu) << 16) /* cap on CTAs, 0 = auto */
 #define KVS_F_GET_MAX_CTAS(f) (((f) >> 16) & 0xFFFFu)
 

@@ -33,12 +33,16 @@
  *   store:     for each chunk j, layer l, kv and head h:
  *                  amax  = max |x| over the finite elements x of the chunk's
  *                          n tokens and D dims of head h (0 if none),
- *                  scale = amax / 448 in binary32 (1 when amax is 0),
- *                  code  = e4m3(x / scale) with x / scale a binary32
- *                          division; the conversion rounds to nearest even
- *                          and saturates (OFP8 saturation mode): magnitudes
- *                          at or beyond 448, and infinities, give +-448; NaN
+ *                  scale = amax / 448 in binary32 (1 when amax is 0), stored,
+ *                  inv   = 448 / amax in binary32 (1 when amax is 0),
+ *                  code  = e4m3(x * inv) with x * inv a binary32 multiply;
+ *                          the conversion rounds to nearest even and
+ *                          saturates (OFP8 saturation mode): magnitudes at
+ *                          or beyond 448, and infinities, give +-448; NaN
  *                          gives the NaN code 0x7F.
+ *              (One division per head and one multiply per element: the
+ *              format is this build's, not the paper's, and a reciprocal
+ *              multiply keeps quantisation cheap next to the bytes it moves.)
  *
  * Every other element is left untouched.  Return values as in kvs_oracle.c:
  * 0, -2 when a token cannot be mapped through the block table, -1 for a
@@ -250,13 +254,14 @@ int kvs_oracle_store_fp8(int L, int H, int D, int B,
                         }
                     }
                     float scale = amax > 0.0f ? amax / 448.0f : 1.0f;
+                    float inv = amax > 0.0f ? 448.0f / amax : 1.0f;
                     put_scale(chunks[j], l, kv, h, H, scale);
                     for (int64_t i = 0; i < n; ++i) {
                         int64_t slot = slot_of(s + i, B, block_table, block_table_len, num_blocks);
                         if (slot < 0) continue;
                         for (int64_t d = 0; d < D; ++d) {
                             float x = kvs_oracle_bf16_value(plane[paged_elem(slot, h, d, H, D)]);
-                            float q = x / scale;                 /* one binary32 division */
+                            float q = x * inv;                   /* one binary32 multiply */
                             codes[chunk_code(l, kv, i, h, d, n, H, D)] = kvs_oracle_e4m3_code(q);
                         }
                     }

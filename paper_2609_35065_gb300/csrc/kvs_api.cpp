@@ -532,11 +532,13 @@ Job make_job(DevState& st, const kvs_geometry* g, const kvs_paged_cache* cache, 
 
 // Internal flavour: the double-buffered kernel used for host-resident chunks.
 constexpr int kKernelLink = 100;
+constexpr int kKernelLinkPrefetch = 101;   // retrieval only
 
 int launch_kernel(const Job& j, int flavour, int vec, int grid, cudaStream_t s) {
     if (j.num_pieces == 0) return KVS_OK;
     cudaError_t e = (flavour == KVS_KERNEL_TMA) ? launch_tma(j, grid, s)
-                  : (flavour == kKernelLink && vec == 16) ? launch_link(j, grid, s)
+                  : (flavour == kKernelLinkPrefetch && vec == 16) ? launch_link_prefetch(j, grid, s)
+                  : ((flavour == kKernelLink || flavour == kKernelLinkPrefetch) && vec == 16) ? launch_link(j, grid, s)
                   : launch_ldg(j, vec, grid, s);
     if (e != cudaSuccess) return fail(KVS_ERR_CUDA, "kernel launch failed: %s", cudaGetErrorString(e));
     ++g_launches;
@@ -835,8 +837,9 @@ int copy_call(const kvs_geometry* g, const kvs_paged_cache* cache, const kvs_req
                 rc = host_variant == KVS_VARIANT_DMA ? run_dma(g, pl, pitch, retrieve, s, host_addr)
                                                      : run_hbmcopy(st, g, cache, pl, u, mode, flavour, grid, s, host_addr);
             } else {
+                const int lf = (retrieve && (flags & KVS_F_PREFETCH_L2)) ? kKernelLinkPrefetch : kKernelLink;
                 rc = launch_kernel(make_job(st, g, cache, pl, u, pl.num_device, pl.num_host, mode, p0, np),
-                                   kKernelLink, vec, host_grid, s);
+                                   lf, vec, host_grid, s);
             }
             if (rc) return rc;
         }
@@ -923,10 +926,13 @@ int fp8_call(const kvs_geometry* g, const kvs_paged_cache* cache, const kvs_requ
         f.heads = (uint32_t)g->num_kv_heads;
         f.head_dim = (uint32_t)g->head_dim;
         f.scale_bytes = (uint32_t)fp8_scale_bytes(g);
+        // floor(2^32 / B) + 1 fits 32 bits for B >= 2; the kernel divides by B = 1 itself
+        f.block_magic = g->block_size >= 2 ? (uint32_t)((1ull << 32) / (uint64_t)g->block_size + 1) : 0;
         return f;
     };
     auto run = [&](const Fp8Job& f, int grid) -> int {
-        cudaError_t e = retrieve ? launch_fp8_retrieve(f, grid, s) : launch_fp8_store(f, grid, s);
+        cudaError_t e = retrieve ? launch_fp8_retrieve(f, grid, s)
+                                 : launch_fp8_store(f, grid, s, (uint32_t)g->chunk_tokens);
         if (e != cudaSuccess) return fail(KVS_ERR_CUDA, "fp8 kernel launch failed: %s", cudaGetErrorString(e));
         ++g_launches;
         return KVS_OK;
@@ -945,7 +951,8 @@ int fp8_call(const kvs_geometry* g, const kvs_paged_cache* cache, const kvs_requ
     if (pl.num_device) {
         const Fp8Job f = fjob(0, pl.num_device);
         if (f.job.num_pieces >= (1ull << 31)) return fail(KVS_ERR_INVALID_ARG, "call too large: split it");
-        rc = run(f, cap);
+        // HBM chunks: uncapped retrievals run one CTA per piece
+        rc = run(f, cap ? cap : (retrieve ? kFp8PerPiece : 0));
         if (rc) return rc;
     }
     if (flags & KVS_F_VALIDATE) {

@@ -11,15 +11,15 @@
 //
 //   retrieve  plane = bf16_rn(fp32(code) *rn scale); a NaN product gives 0x7FFF
 //   store     per (chunk, layer, K/V, head): amax over the finite elements,
-//             scale = amax /rn 448 (1 when amax is 0), code = e4m3 of
-//             x /rn scale, rounded to nearest even and saturated at +-448;
-//             NaN gives the code 0x7F
+//             scale = amax /rn 448 (stored), inv = 448 /rn amax (both 1 when
+//             amax is 0), code = e4m3 of x *rn inv, rounded to nearest even
+//             and saturated at +-448; NaN gives the code 0x7F
 //
 // Every element conversion uses the hardware conversions of sm_89+ (E4M3 <->
-// f16 pairs, f32 -> bf16 pairs) and IEEE round-to-nearest multiply / divide;
-// NaN results and magnitudes at or below 2^-10 (which round to zero) are set
-// explicitly, so the result does not depend on how a conversion treats NaN
-// signs or binary32 subnormals.
+// f16 pairs, f32 -> bf16 / E4M3 pairs, round to nearest even, the E4M3 one
+// saturating) and IEEE round-to-nearest multiplies; NaN results are set to
+// one canonical pattern explicitly (0x7FFF for BF16, 0x7F for E4M3), so the
+// result does not depend on how a conversion treats a NaN's sign.
 //
 // Retrieval is bound by the host link (or HBM for device chunks): a persistent
 // grid of 128-thread CTAs walks 16 KiB pieces of codes; each thread keeps two
@@ -194,48 +194,134 @@ __global__ void __launch_bounds__(kRtThreads) kvs_fp8_retrieve_kernel(const Fp8J
     }
 }
 
+// Device chunks (HBM source): one CTA per piece, no persistence; the launch
+// bound keeps the kernel at 64 registers so eight CTAs -- 128 KiB of code
+// loads -- are in flight per SM, and the hardware block scheduler overlaps one
+// CTA's stores with the next CTA's loads.
+__global__ void __launch_bounds__(kRtThreads, 8) kvs_fp8_retrieve_piece_kernel(const Fp8Job f) {
+    __shared__ float sm_scale[kFp8MaxHeads];
+    Fp8Piece pc;
+    if (!fp8_piece(f, blockIdx.x, pc)) return;         // uniform across the CTA
+    RtRegs r;
+    rt_load(f, pc, r);
+    rt_store(f, pc, r, sm_scale);
+}
+
 // ---------------------------------------------------------------------------
 // Store-back (quantise)
 // ---------------------------------------------------------------------------
 
-// Largest |x| bit pattern among the finite BF16 values of a 16-byte vector
-// (|x| of a finite BF16 orders like its bits with the sign cleared).
+// Per-halfword running maximum of |x| over the finite BF16 values of a
+// 32-bit word pair (|x| of a finite BF16 orders like its bits with the sign
+// cleared; infinities and NaN, exponent all ones, count as 0).
+__device__ __forceinline__ uint32_t amax2(uint32_t m2, uint32_t w) {
+    const uint32_t a = w & 0x7FFF7FFFu;
+    return __vmaxu2(m2, a & ~__vcmpgeu2(a, 0x7F807F80u));
+}
+
 __device__ __forceinline__ uint32_t amax_bits8(const uint4& v) {
-    uint32_t m = 0;
-    const uint32_t w[4] = {v.x, v.y, v.z, v.w};
-#pragma unroll
-    for (int k = 0; k < 4; ++k) {
-        const uint32_t a = w[k] & 0x7FFFu, b = (w[k] >> 16) & 0x7FFFu;
-        if (a < 0x7F80u) m = max(m, a);
-        if (b < 0x7F80u) m = max(m, b);
-    }
-    return m;
+    uint32_t m2 = amax2(amax2(amax2(amax2(0u, v.x), v.y), v.z), v.w);
+    return max(m2 & 0xFFFFu, m2 >> 16);
 }
 
 __device__ __forceinline__ float bf16_lo(uint32_t w) { return __uint_as_float(w << 16); }
 __device__ __forceinline__ float bf16_hi(uint32_t w) { return __uint_as_float(w & 0xFFFF0000u); }
 
-// One E4M3 code of q: NaN -> 0x7F; |q| <= 2^-10 rounds to a signed zero; the
-// rest through the saturating round-to-nearest-even conversion.
-__device__ __forceinline__ uint32_t fix_code(float q, uint32_t hw) {
-    if (q != q) return 0x7Fu;
-    if (fabsf(q) <= 0x1p-10f) return (__float_as_uint(q) >> 24) & 0x80u;
-    return hw;
+// Two BF16 (one word) times `inv` -> two E4M3 codes (saturating, nearest even).
+__device__ __forceinline__ uint32_t e4m3x2_of(uint32_t w, float inv) {
+    return (uint32_t)__nv_cvt_float2_to_fp8x2(make_float2(__fmul_rn(bf16_lo(w), inv), __fmul_rn(bf16_hi(w), inv)),
+                                              __NV_SATFINITE, __NV_E4M3);
 }
 
-__device__ __forceinline__ uint32_t e4m3x2(float a, float b) {
-    const uint32_t hw = (uint32_t)__nv_cvt_float2_to_fp8x2(make_float2(a, b), __NV_SATFINITE, __NV_E4M3);
-    return fix_code(a, hw & 0xFFu) | (fix_code(b, hw >> 8) << 8);
+// Four codes per word: every NaN code (S.1111.111) becomes 0x7F.
+__device__ __forceinline__ uint32_t canon_nan4(uint32_t c) {
+    const uint32_t nan = __vcmpeq4(c & 0x7F7F7F7Fu, 0x7F7F7F7Fu);
+    return (c & ~nan) | (0x7F7F7F7Fu & nan);
 }
 
-// 16 BF16 (two vectors) divided by `s` -> 16 codes.
-__device__ __forceinline__ uint4 quant16(const uint4& a, const uint4& b, float s) {
-    const uint32_t w[8] = {a.x, a.y, a.z, a.w, b.x, b.y, b.z, b.w};
-    uint32_t c[8];
+// 8 BF16 (one 16-byte vector) -> 8 codes.
+__device__ __forceinline__ uint2 quant8(const uint4& a, float inv) {
+    return make_uint2(canon_nan4(e4m3x2_of(a.x, inv) | (e4m3x2_of(a.y, inv) << 16)),
+                      canon_nan4(e4m3x2_of(a.z, inv) | (e4m3x2_of(a.w, inv) << 16)));
+}
+
+// 16 BF16 (two vectors) -> 16 codes.
+__device__ __forceinline__ uint4 quant16(const uint4& a, const uint4& b, float inv) {
+    const uint2 x = quant8(a, inv), y = quant8(b, inv);
+    return make_uint4(x.x, x.y, y.x, y.y);
+}
+
+__device__ __forceinline__ void st_cs8(uint64_t a, const uint2& v) {
+    asm volatile("st.global.cs.v2.u32 [%0], {%1,%2};" :: "l"(a), "r"(v.x), "r"(v.y) : "memory");
+}
+
+// Single pass, one CTA per (entry, plane, head): the head's n x D BF16 elements
+// of the chunk (at most kHeadVec * kStThreads * 8, i.e. 64 KiB) are loaded
+// into registers at once (kHeadVec 16-byte vectors per thread, all in flight),
+// reduced to the head's amax across the CTA, and quantised from registers:
+// the planes are read once and the loads of a whole head are in flight together.
+// Thread t handles the 16-byte column w = t % (D/8) of tokens t / (D/8) + u *
+// step (step = kStThreads / (D/8) tokens), so the column, and with it the
+// address arithmetic inside a token row, is fixed per thread.  Needs D/8 to
+// divide kStThreads and n, B below 2^16 (checked by the launcher).
+constexpr int kHeadVec = 16;
+constexpr uint32_t kHeadMaxElems = kHeadVec * kStThreads * 8;
+
+__global__ void __launch_bounds__(kStThreads) kvs_fp8_store_head_kernel(const Fp8Job f, uint32_t num_segments) {
+    __shared__ uint32_t warp_max[kStThreads / 32];
+    __shared__ float sm_inv;
+    const Job& j = f.job;
+    const uint32_t H = f.heads, D = f.head_dim, vpt = D / 8;       // 16-byte vectors per token row of a head
+    const uint32_t B = j.block_size, step = kStThreads / vpt;
+    const uint32_t w = threadIdx.x % vpt, i0 = threadIdx.x / vpt;
+    const uint64_t row2 = (uint64_t)H * D * 2;                       // BF16 bytes per token row
+    for (uint32_t seg = blockIdx.x; seg < num_segments; seg += gridDim.x) {
+        const uint32_t eh = seg / H, h = seg - eh * H;
+        const uint32_t e = eh / j.num_planes;
+        const uint32_t p = j.plane_begin + (eh - e * j.num_planes);
+        const Entry en = j.entries[e];
+        const uint32_t n = (uint32_t)en.n_tok;
+        const int32_t* blocks = j.blocks + (size_t)(j.entry_base + e) * j.blocks_per_chunk;
+        const uint64_t src0 = j.planes[p] + (uint64_t)h * D * 2 + (uint64_t)w * 16;
+        uint4 v[kHeadVec];
+        uint32_t m2 = 0;
+        bool bad = false;
 #pragma unroll
-    for (int k = 0; k < 8; ++k)
-        c[k] = e4m3x2(__fdiv_rn(bf16_lo(w[k]), s), __fdiv_rn(bf16_hi(w[k]), s));
-    return make_uint4(c[0] | (c[1] << 16), c[2] | (c[3] << 16), c[4] | (c[5] << 16), c[6] | (c[7] << 16));
+        for (int u = 0; u < kHeadVec; ++u) {
+            const uint32_t i = i0 + u * step;
+            v[u] = make_uint4(0, 0, 0, 0);
+            if (i < n) {
+                const uint32_t bi = B == 1 ? i : __umulhi(i, f.block_magic), r = i - bi * B;
+                const int32_t blk = __ldg(blocks + bi);
+                if (blk < 0 || blk >= j.num_blocks) bad = true;
+                else v[u] = ld_nc16(src0 + ((uint64_t)blk * B + r) * row2);
+            }
+        }
+#pragma unroll
+        for (int u = 0; u < kHeadVec; ++u)
+            m2 = amax2(amax2(amax2(amax2(m2, v[u].x), v[u].y), v[u].z), v[u].w);
+        if (bad) atomicCAS(j.err, 0, KVS_ERR_BOUNDS);
+        const uint32_t m = __reduce_max_sync(0xFFFFFFFFu, max(m2 & 0xFFFFu, m2 >> 16));
+        if ((threadIdx.x & 31) == 0) warp_max[threadIdx.x >> 5] = m;
+        __syncthreads();
+        uint32_t a = 0;
+        for (int k = 0; k < kStThreads / 32; ++k) a = max(a, warp_max[k]);
+        if (threadIdx.x == 0) {
+            const float af = __uint_as_float(a << 16);
+            const float sc = af > 0.0f ? __fdiv_rn(af, 448.0f) : 1.0f;
+            sm_inv = af > 0.0f ? __fdiv_rn(448.0f, af) : 1.0f;
+            *reinterpret_cast<float*>(en.chunk + ((uint64_t)p * H + h) * 4) = sc;
+        }
+        __syncthreads();
+        const float inv = sm_inv;
+        const uint64_t codes = en.chunk + f.scale_bytes + (uint64_t)p * n * H * D + (uint64_t)h * D + (uint64_t)w * 8;
+#pragma unroll
+        for (int u = 0; u < kHeadVec; ++u) {
+            const uint32_t i = i0 + u * step;
+            if (i < n) st_cs8(codes + (uint64_t)i * H * D, quant8(v[u], inv));
+        }
+        __syncthreads();                                   // warp_max / sm_inv are reused
+    }
 }
 
 constexpr int kStUnroll = 4;                         // vectors per thread in flight per step
@@ -243,7 +329,7 @@ constexpr int kStUnroll = 4;                         // vectors per thread in fl
 // One CTA per (entry, plane) segment: the chunk's n tokens of that plane.
 __global__ void __launch_bounds__(kStThreads) kvs_fp8_store_kernel(const Fp8Job f, uint32_t num_segments) {
     __shared__ uint32_t amax[kFp8MaxHeads];
-    __shared__ float scale[kFp8MaxHeads];
+    __shared__ float scale[kFp8MaxHeads];                    // holds 448 / amax per head
     const Job& j = f.job;
     const uint32_t H = f.heads, vph = f.head_dim / 16, vpr = H * vph;
     const uint64_t row2 = (uint64_t)H * f.head_dim * 2;          // BF16 bytes per token row
@@ -306,7 +392,7 @@ __global__ void __launch_bounds__(kStThreads) kvs_fp8_store_kernel(const Fp8Job 
         for (uint32_t h = threadIdx.x; h < H; h += blockDim.x) {
             const float a = __uint_as_float(amax[h] << 16);
             const float s = a > 0.0f ? __fdiv_rn(a, 448.0f) : 1.0f;
-            scale[h] = s;
+            scale[h] = a > 0.0f ? __fdiv_rn(448.0f, a) : 1.0f;        // the inverse, for pass 2
             *reinterpret_cast<float*>(en.chunk + ((uint64_t)p * H + h) * 4) = s;
         }
         __syncthreads();
@@ -353,6 +439,10 @@ int sm_count() {
 cudaError_t launch_fp8_retrieve(const Fp8Job& fj, int grid, cudaStream_t s) {
     const uint64_t n = fj.job.num_pieces;
     if (n == 0) return cudaSuccess;
+    if (grid == kFp8PerPiece) {
+        kvs_fp8_retrieve_piece_kernel<<<(uint32_t)n, kRtThreads, 0, s>>>(fj);
+        return cudaGetLastError();
+    }
     int per_sm = 0;
     cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, kvs_fp8_retrieve_kernel, kRtThreads, 0);
     const int full = sm_count() * std::max(per_sm, 1);
@@ -362,7 +452,16 @@ cudaError_t launch_fp8_retrieve(const Fp8Job& fj, int grid, cudaStream_t s) {
     return cudaGetLastError();
 }
 
-cudaError_t launch_fp8_store(const Fp8Job& fj, int grid, cudaStream_t s) {
+cudaError_t launch_fp8_store(const Fp8Job& fj, int grid, cudaStream_t s, uint32_t chunk_tokens) {
+    const uint32_t vpt = fj.head_dim / 8;
+    if ((uint64_t)chunk_tokens * fj.head_dim <= kHeadMaxElems && kStThreads % vpt == 0 && chunk_tokens < 65536 &&
+        fj.job.block_size < 65536) {
+        const uint64_t segs = (uint64_t)fj.job.num_entries * fj.job.num_planes * fj.heads;
+        if (segs == 0) return cudaSuccess;
+        if (grid <= 0 || (uint64_t)grid > segs) grid = (int)std::min<uint64_t>(segs, 1u << 30);
+        kvs_fp8_store_head_kernel<<<grid, kStThreads, 0, s>>>(fj, (uint32_t)segs);
+        return cudaGetLastError();
+    }
     const uint64_t segs = (uint64_t)fj.job.num_entries * fj.job.num_planes;
     if (segs == 0) return cudaSuccess;
     if (grid <= 0 || (uint64_t)grid > segs) grid = (int)segs;

@@ -55,6 +55,8 @@ cudaError_t launch_ldg(const Job& job, int vec_bytes, int grid, cudaStream_t s);
 cudaError_t launch_tma(const Job& job, int grid, cudaStream_t s);
 // Double-buffered 16-byte flavour for host-resident chunks (retrieve or store).
 cudaError_t launch_link(const Job& job, int grid, cudaStream_t s);
+// The same for retrieval, with each CTA's upcoming pieces prefetched into L2.
+cudaError_t launch_link_prefetch(const Job& job, int grid, cudaStream_t s);
 // Contiguous copy of `bytes` (multiple of 16, 16-byte aligned) for bandwidth probes.
 cudaError_t launch_flat_copy(void* dst, const void* src, uint64_t bytes, int grid, cudaStream_t s);
 // Layer-wise copy of host chunks in one launch: pieces go in plane-major
@@ -80,13 +82,18 @@ struct Fp8Job {
     uint32_t heads;              // H
     uint32_t head_dim;           // D, a multiple of 16
     uint32_t scale_bytes;        // bytes of the scale block, a multiple of 256
+    uint32_t block_magic;        // floor(2^32 / B) + 1: floor(i / B) = umulhi(i, magic) for i, B < 2^16
 };
 constexpr uint32_t kFp8MaxHeads = 128;
 // Retrieval: a persistent grid of `grid` CTAs (<= 0: fill the GPU) over pieces of at
-// most 16 KiB of codes, double-buffered; the number of pieces is in job.num_pieces.
+// most 16 KiB of codes, double-buffered; grid == kFp8PerPiece: one CTA per piece
+// (HBM sources).  The number of pieces is in job.num_pieces.
+constexpr int kFp8PerPiece = -1;
 cudaError_t launch_fp8_retrieve(const Fp8Job& fj, int grid, cudaStream_t s);
-// Store-back: one CTA per (entry, plane), or a grid-stride loop over them with `grid` > 0.
-cudaError_t launch_fp8_store(const Fp8Job& fj, int grid, cudaStream_t s);
+// Store-back: one CTA per (entry, plane, head) in a single pass when a head's
+// chunk_tokens x head_dim elements fit the CTA's registers, else one CTA per
+// (entry, plane) in two passes; a grid-stride loop over them with `grid` > 0.
+cudaError_t launch_fp8_store(const Fp8Job& fj, int grid, cudaStream_t s, uint32_t chunk_tokens);
 // Codes per retrieval piece (16 KiB).
 constexpr uint32_t kFp8PieceCodes = 16384;
 

@@ -280,6 +280,59 @@ __global__ void __launch_bounds__(kLdgThreads) kvs_link_kernel(const Decoder dc,
     }
 }
 
+// L2-prefetch flavour of the host-link retrieval.  Over the host link a piece's
+// loads take ~15 us beside a busy GPU, so the plain flavour needs ~3 MiB of
+// loads in flight, held in registers: 16 or more SMs' worth of CTAs.  Here the
+// CTA's thread 0 keeps the CTA's next `ahead` pieces in flight as bulk L2
+// prefetches (cp.async.bulk.prefetch.L2, which holds no registers or shared
+// memory), so the bytes in flight wait in L2; the CTA's own loads then find
+// their piece in L2 and the grid can be small.  Prefetches of a piece that
+// are still in flight, or evicted, only cost time: the loads fetch the bytes
+// themselves either way.
+__device__ __forceinline__ void prefetch_l2(uint64_t addr, uint32_t bytes) {
+    asm volatile("cp.async.bulk.prefetch.L2.global [%0], %1;" :: "l"(addr), "r"(bytes) : "memory");
+}
+
+__device__ __forceinline__ bool next_piece_pf(const Decoder& dc, uint32_t num_pieces, uint32_t stride_ahead,
+                                              uint32_t& q, Piece& pc) {
+    while (q < num_pieces) {
+        const uint32_t cur = q;
+        q += gridDim.x;
+        if (threadIdx.x == 0) {
+            const uint32_t f = cur + stride_ahead;            // < 2^32: both terms are below 2^31
+            Piece pf;
+            if (f < num_pieces && decode_piece(dc, f, pf)) prefetch_l2(pf.chunk_addr, pf.len);
+        }
+        if (decode_piece(dc, cur, pc)) return true;
+    }
+    return false;
+}
+
+__global__ void __launch_bounds__(kLdgThreads) kvs_link_pf_kernel(const Decoder dc, uint32_t num_pieces,
+                                                                  uint32_t ahead) {
+    const uint32_t stride_ahead = ahead * gridDim.x;
+    if (threadIdx.x == 0)
+        for (uint32_t k = 0; k < ahead; ++k) {
+            const uint32_t f = blockIdx.x + k * gridDim.x;
+            Piece pf;
+            if (f < num_pieces && decode_piece(dc, f, pf)) prefetch_l2(pf.chunk_addr, pf.len);
+        }
+    uint4 ra[kLdgUnroll], rb[kLdgUnroll];
+    Piece pa, pb;
+    uint32_t q = blockIdx.x;
+    bool ha = next_piece_pf(dc, num_pieces, stride_ahead, q, pa);
+    if (ha) load_piece16(pa.chunk_addr, pa.len, ra);
+    while (ha) {
+        const bool hb = next_piece_pf(dc, num_pieces, stride_ahead, q, pb);
+        if (hb) load_piece16(pb.chunk_addr, pb.len, rb);
+        store_piece16(pa.plane_addr, pa.len, ra);
+        if (!hb) break;
+        ha = next_piece_pf(dc, num_pieces, stride_ahead, q, pa);
+        if (ha) load_piece16(pa.chunk_addr, pa.len, ra);
+        store_piece16(pb.plane_addr, pb.len, rb);
+    }
+}
+
 // Plane-major decode for the signalling kernel: q -> (plane, entry, block, piece).
 __device__ __forceinline__ bool decode_piece_plane_major(const Decoder& dc, const FastDiv& entries, uint32_t q,
                                                          uint32_t& p_rel, Piece& pc) {
@@ -609,6 +662,15 @@ int link_ctas_per_sm() {
         if (n <= 0) n = 1;
     }
     return n;
+}
+
+cudaError_t launch_link_prefetch(const Job& job, int grid, cudaStream_t s) {
+    if (job.num_pieces == 0) return cudaSuccess;
+    grid = clamp_grid(grid, link_ctas_per_sm(), job.num_pieces);
+    // about 4 MiB of prefetches in flight over the whole grid
+    const uint32_t ahead = (uint32_t)std::min(64, std::max(2, (int)((4u << 20) / kPieceBytes) / grid));
+    kvs_link_pf_kernel<<<grid, kLdgThreads, 0, s>>>(make_decoder(job), (uint32_t)job.num_pieces, ahead);
+    return cudaGetLastError();
 }
 
 cudaError_t launch_link(const Job& job, int grid, cudaStream_t s) {

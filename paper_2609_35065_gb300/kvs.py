@@ -45,6 +45,7 @@ KVS_F_NO_DEDUP = 1 << 5
 KVS_F_LAYER_LAUNCHES = 1 << 6
 KVS_F_LAYER_SIGNAL = 1 << 7
 KVS_F_FORCE_DMA = 1 << 8
+KVS_F_PREFETCH_L2 = 1 << 9
 KVS_DIR_RETRIEVE = 0
 KVS_DIR_STORE = 1
 

@@ -178,7 +178,9 @@ def _fancy_store(L, H, D, B, planes, first, chunks, ntok, table, lib):
         fin = np.where(np.isfinite(x), np.abs(x), np.float32(0))
         amax = fin.max(axis=(1, 3)).astype(np.float32)                                           # [2L][H]
         scale = np.where(amax > 0, amax / np.float32(448), np.float32(1)).astype(np.float32)
-        q = (x / scale[:, None, :, None]).astype(np.float32)
+        with np.errstate(divide="ignore"):
+            inv = np.where(amax > 0, np.float32(448) / amax, np.float32(1)).astype(np.float32)
+        q = (x * inv[:, None, :, None]).astype(np.float32)
         q = np.where(np.isnan(q), q, np.clip(q, -448, 448)).astype(np.float32).reshape(-1)
         c[:2 * L * H * 4] = scale.reshape(-1).view(np.uint8)
         c[hdr:] = np.where(np.isnan(q), np.uint8(0x7F), _torch_encode(q))
@@ -240,7 +242,7 @@ def pin_fp8_fancy(lib):
 
 def pin_fp8_exact_tags(lib):
     """Per head, values are E4M3 values times 2^k_h with the head's maximum at exactly
-    448 * 2^k_h, so scale = 2^k_h and every conversion is exact."""
+    448 * 2^k_h, so scale = 2^k_h, inv = 2^-k_h and every conversion is exact."""
     rng = np.random.default_rng(11)
     for L, H, D, B, first, ntok in [(2, 3, 16, 4, 0, [8, 8, 5]), (1, 2, 32, 1, 8, [8, 3]),
                                     (3, 1, 16, 16, 32, [32, 32])]:

@@ -145,3 +145,20 @@ def test_fp8_refusals():
     assert ei.value.code == kvs.KVS_ERR_UNSUPPORTED
     torch.cuda.synchronize()
     assert torch.all(buf.planes == buf.planes.view(-1)[0])
+
+
+@pytest.mark.parametrize("residency", ["host", "device"])
+def test_fp8_store_two_pass_for_large_heads(residency):
+    """chunk_tokens x head_dim above what one CTA holds in registers (256 x 256 = 65,536
+    elements per head): the store takes the two-pass kernel (one CTA per chunk and plane);
+    a ragged last chunk and a partial last block included."""
+    w = synth.custom(2, 2, 256, 16, 256, 120, [700, 300], [0, 0], seed=9, residency=residency,
+                     store_tokens=[700, 300])
+    buf = buffers.allocate_fp8(w, store=True, store_residency=residency)
+    rng = torch.Generator(device="cuda").manual_seed(9)
+    for p in range(buf.planes.shape[0]):
+        synth.fill_values(buf.planes[p], "normal", rng)
+    torch.cuda.synchronize()
+    _store(buf)
+    torch.cuda.synchronize()
+    gc.check_store_fp8(buf)

@@ -157,3 +157,31 @@ def test_tune_argument_checks():
     before = kvs.kvs_get_choice()["chosen_retrieve_host"]
     rep = kvs.kvs_tune(w2.geom, b2.plane_ptrs, w2.num_blocks, b2.requests, None, 0, 0, 1)
     assert rep["host_bytes"] == 0 and rep["chosen"] == before
+
+
+@pytest.mark.parametrize("cap", [0, 3, 12], ids=["default_grid", "3_ctas", "12_ctas"])
+def test_prefetch_l2_retrieval(cap):
+    """Host-link retrieval with L2 prefetches of each CTA's upcoming pieces: the 8B shape
+    (2 requests, 512 MiB) and the ragged multi-piece shape, every element checked."""
+    flags = kvs.KVS_F_PREFETCH_L2 | kvs.KVS_F_VALIDATE | kvs.KVS_F_MAX_CTAS(cap)
+    for w in (synth.llama8b(requests=2, num_blocks=1024),
+              synth.custom(2, 8, 256, 16, 256, 300, [1024, 700, 512], [1024, 700, 512], seed=5, dist="normal")):
+        buf = buffers.allocate(w)
+        kvs.kvs_retrieve(w.geom, buf.plane_ptrs, w.num_blocks, buf.requests, None, flags)
+        torch.cuda.synchronize()
+        gc.check_retrieve(buf)
+        gc.free(buf)
+
+
+@pytest.mark.parametrize("seed", range(8))
+def test_prefetch_l2_random_small_geometries(seed):
+    """Random geometries: 16-byte rows take the prefetching kernel, the rest the vector
+    kernel; stores ignore the flag."""
+    w = gc.random_workload(seed)
+    buf = buffers.allocate(w, store=True, store_residency="host")
+    flags = kvs.KVS_F_PREFETCH_L2 | kvs.KVS_F_VALIDATE | kvs.KVS_F_MAX_CTAS(seed % 3)
+    kvs.kvs_retrieve(w.geom, buf.plane_ptrs, w.num_blocks, buf.requests, None, flags)
+    kvs.kvs_store(w.geom, buf.plane_ptrs, w.num_blocks, buf.store_requests, None, flags)
+    torch.cuda.synchronize()
+    gc.check_retrieve(buf)
+    gc.check_store(buf)

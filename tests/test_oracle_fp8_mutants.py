@@ -36,7 +36,10 @@ MUTANTS = {
                                "if (!isnan(x) && fabsf(x) > amax) amax = fabsf(x);"),
     "scale_divisor_wrong": ("float scale = amax > 0.0f ? amax / 448.0f : 1.0f;",
                             "float scale = amax > 0.0f ? amax / 240.0f : 1.0f;"),
-    "store_multiplies": ("float q = x / scale;", "float q = x * scale;"),
+    "inverse_wrong": ("float inv = amax > 0.0f ? 448.0f / amax : 1.0f;",
+                      "float inv = amax > 0.0f ? 447.0f / amax : 1.0f;"),
+    "store_uses_scale_not_inverse": ("float q = x * inv;", "float q = x * scale;"),
+    "store_divides_by_inverse": ("float q = x * inv;", "float q = x / inv;"),
     "retrieve_ignores_scale": ("float y = x * scale;", "float y = x;"),
     "negative_zero_lost": ("uint8_t sign = signbit(v) ? 0x80 : 0x00;", "uint8_t sign = v < 0 ? 0x80 : 0x00;"),
 }
