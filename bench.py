@@ -883,7 +883,7 @@ def default_line_legs(args, buf, bw, stream, sampler, flags):
                    "store": {"link_gbs": round(fbytes / ssec / 1e9, 2),
                              "frac_of_d2h_link": round(fbytes / ssec / 1e9 / d2h_peak, 4),
                              "tokens_per_s": round(w.matched_tokens / ssec, 1),
-                             "kernel": "kvs_fp8_store_kernel", "clocks": sampler.summary(*swin)},
+                             "kernel": "kvs_fp8_store_head_kernel", "clocks": sampler.summary(*swin)},
                    "chunk_bytes": fbytes, "format": "OCP OFP8 rev 1.0 E4M3 codes + binary32 scale per "
                                                     "(chunk, layer, K/V, head)", "calls": n}
     del fb

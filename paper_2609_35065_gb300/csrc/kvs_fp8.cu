@@ -17,9 +17,10 @@
 //
 // Every element conversion uses the hardware conversions of sm_89+ (E4M3 <->
 // f16 pairs, f32 -> bf16 / E4M3 pairs, round to nearest even, the E4M3 one
-// saturating) and IEEE round-to-nearest multiplies; NaN results are set to
-// one canonical pattern explicitly (0x7FFF for BF16, 0x7F for E4M3), so the
-// result does not depend on how a conversion treats a NaN's sign.
+// saturating) and IEEE round-to-nearest multiplies.  A NaN product is set to
+// 0x7FFF explicitly on retrieval; on store, the saturating E4M3 conversion
+// itself gives 0x7F for every NaN input, either sign (the special-values
+// parity test plants both and compares with the oracle).
 //
 // Retrieval is bound by the host link (or HBM for device chunks): a persistent
 // grid of 128-thread CTAs walks 16 KiB pieces of codes; each thread keeps two
@@ -27,10 +28,11 @@
 // loads are in flight while the current one is converted and stored.  The H
 // scales of a piece's plane are loaded once per piece by H threads (one 4-byte
 // load each, beside the codes) and shared through shared memory, instead of
-// one scale load per vector.  Store-back runs one 256-thread CTA per (chunk,
-// plane) over the whole GPU: a first pass takes the per-head amax, a second
-// quantises (the re-read hits L2 or HBM; the destination write over the host
-// link is the bound); both passes keep four vectors per thread in flight.
+// one scale load per vector; HBM chunks run one CTA per piece instead.
+// Store-back runs one 256-thread CTA per (chunk, plane, head): the head's BF16
+// elements are loaded into registers at once, reduced to the amax and
+// quantised from registers (heads too large for that take a two-pass kernel,
+// one CTA per (chunk, plane)).
 #include <cuda_bf16.h>
 #include <cuda_fp16.h>
 #include <cuda_fp8.h>
@@ -233,16 +235,10 @@ __device__ __forceinline__ uint32_t e4m3x2_of(uint32_t w, float inv) {
                                               __NV_SATFINITE, __NV_E4M3);
 }
 
-// Four codes per word: every NaN code (S.1111.111) becomes 0x7F.
-__device__ __forceinline__ uint32_t canon_nan4(uint32_t c) {
-    const uint32_t nan = __vcmpeq4(c & 0x7F7F7F7Fu, 0x7F7F7F7Fu);
-    return (c & ~nan) | (0x7F7F7F7Fu & nan);
-}
-
 // 8 BF16 (one 16-byte vector) -> 8 codes.
 __device__ __forceinline__ uint2 quant8(const uint4& a, float inv) {
-    return make_uint2(canon_nan4(e4m3x2_of(a.x, inv) | (e4m3x2_of(a.y, inv) << 16)),
-                      canon_nan4(e4m3x2_of(a.z, inv) | (e4m3x2_of(a.w, inv) << 16)));
+    return make_uint2(e4m3x2_of(a.x, inv) | (e4m3x2_of(a.y, inv) << 16),
+                      e4m3x2_of(a.z, inv) | (e4m3x2_of(a.w, inv) << 16));
 }
 
 // 16 BF16 (two vectors) -> 16 codes.
@@ -267,60 +263,76 @@ __device__ __forceinline__ void st_cs8(uint64_t a, const uint2& v) {
 constexpr int kHeadVec = 16;
 constexpr uint32_t kHeadMaxElems = kHeadVec * kStThreads * 8;
 
+// One segment of the store: FULL when every thread's kHeadVec vectors all lie in
+// the chunk (n * D/8 == kHeadVec * kStThreads, e.g. a 256-token chunk of head_dim
+// 128), so the loads and stores need no per-vector bounds test.
+template <bool FULL>
+__device__ __forceinline__ void store_head_segment(const Fp8Job& f, uint32_t e, uint32_t p, uint32_t h,
+                                                   uint32_t* warp_max, float* sm_inv) {
+    const Job& j = f.job;
+    const uint32_t H = f.heads, D = f.head_dim, vpt = D / 8;
+    const uint32_t B = j.block_size, step = kStThreads / vpt;
+    const uint32_t w = threadIdx.x % vpt, i0 = threadIdx.x / vpt;
+    const uint64_t row2 = (uint64_t)H * D * 2;
+    const Entry en = j.entries[e];
+    const uint32_t n = (uint32_t)en.n_tok;
+    const int32_t* blocks = j.blocks + (size_t)(j.entry_base + e) * j.blocks_per_chunk;
+    const uint64_t src0 = j.planes[p] + (uint64_t)h * D * 2 + (uint64_t)w * 16;
+    uint4 v[kHeadVec];
+    uint32_t m2 = 0;
+    bool bad = false;
+#pragma unroll
+    for (int u = 0; u < kHeadVec; ++u) {
+        const uint32_t i = i0 + u * step;
+        v[u] = make_uint4(0, 0, 0, 0);
+        if (FULL || i < n) {
+            const uint32_t bi = B == 1 ? i : __umulhi(i, f.block_magic), r = i - bi * B;
+            const int32_t blk = __ldg(blocks + bi);
+            if (blk < 0 || blk >= j.num_blocks) bad = true;
+            else v[u] = ld_nc16(src0 + ((uint64_t)blk * B + r) * row2);
+        }
+    }
+#pragma unroll
+    for (int u = 0; u < kHeadVec; ++u)
+        m2 = amax2(amax2(amax2(amax2(m2, v[u].x), v[u].y), v[u].z), v[u].w);
+    if (bad) atomicCAS(j.err, 0, KVS_ERR_BOUNDS);
+    const uint32_t m = __reduce_max_sync(0xFFFFFFFFu, max(m2 & 0xFFFFu, m2 >> 16));
+    if ((threadIdx.x & 31) == 0) warp_max[threadIdx.x >> 5] = m;
+    __syncthreads();
+    if (threadIdx.x == 0) {
+        uint32_t a = 0;
+        for (int k = 0; k < kStThreads / 32; ++k) a = max(a, warp_max[k]);
+        const float af = __uint_as_float(a << 16);
+        const float sc = af > 0.0f ? __fdiv_rn(af, 448.0f) : 1.0f;
+        *sm_inv = af > 0.0f ? __fdiv_rn(448.0f, af) : 1.0f;
+        *reinterpret_cast<float*>(en.chunk + ((uint64_t)p * H + h) * 4) = sc;
+    }
+    __syncthreads();
+    const float inv = *sm_inv;
+    const uint64_t hd = (uint64_t)H * D;
+    const uint64_t codes = en.chunk + f.scale_bytes + (uint64_t)p * n * hd + (uint64_t)h * D + (uint64_t)w * 8 +
+                           (uint64_t)i0 * hd;
+#pragma unroll
+    for (int u = 0; u < kHeadVec; ++u) {
+        const uint32_t i = i0 + u * step;
+        if (FULL || i < n) st_cs8(codes + (uint64_t)(u * step) * hd, quant8(v[u], inv));
+    }
+    __syncthreads();                                       // warp_max / sm_inv are reused
+}
+
 __global__ void __launch_bounds__(kStThreads) kvs_fp8_store_head_kernel(const Fp8Job f, uint32_t num_segments) {
     __shared__ uint32_t warp_max[kStThreads / 32];
     __shared__ float sm_inv;
     const Job& j = f.job;
-    const uint32_t H = f.heads, D = f.head_dim, vpt = D / 8;       // 16-byte vectors per token row of a head
-    const uint32_t B = j.block_size, step = kStThreads / vpt;
-    const uint32_t w = threadIdx.x % vpt, i0 = threadIdx.x / vpt;
-    const uint64_t row2 = (uint64_t)H * D * 2;                       // BF16 bytes per token row
+    const uint32_t H = f.heads, full_n = kHeadVec * kStThreads / (f.head_dim / 8);
     for (uint32_t seg = blockIdx.x; seg < num_segments; seg += gridDim.x) {
         const uint32_t eh = seg / H, h = seg - eh * H;
         const uint32_t e = eh / j.num_planes;
         const uint32_t p = j.plane_begin + (eh - e * j.num_planes);
-        const Entry en = j.entries[e];
-        const uint32_t n = (uint32_t)en.n_tok;
-        const int32_t* blocks = j.blocks + (size_t)(j.entry_base + e) * j.blocks_per_chunk;
-        const uint64_t src0 = j.planes[p] + (uint64_t)h * D * 2 + (uint64_t)w * 16;
-        uint4 v[kHeadVec];
-        uint32_t m2 = 0;
-        bool bad = false;
-#pragma unroll
-        for (int u = 0; u < kHeadVec; ++u) {
-            const uint32_t i = i0 + u * step;
-            v[u] = make_uint4(0, 0, 0, 0);
-            if (i < n) {
-                const uint32_t bi = B == 1 ? i : __umulhi(i, f.block_magic), r = i - bi * B;
-                const int32_t blk = __ldg(blocks + bi);
-                if (blk < 0 || blk >= j.num_blocks) bad = true;
-                else v[u] = ld_nc16(src0 + ((uint64_t)blk * B + r) * row2);
-            }
-        }
-#pragma unroll
-        for (int u = 0; u < kHeadVec; ++u)
-            m2 = amax2(amax2(amax2(amax2(m2, v[u].x), v[u].y), v[u].z), v[u].w);
-        if (bad) atomicCAS(j.err, 0, KVS_ERR_BOUNDS);
-        const uint32_t m = __reduce_max_sync(0xFFFFFFFFu, max(m2 & 0xFFFFu, m2 >> 16));
-        if ((threadIdx.x & 31) == 0) warp_max[threadIdx.x >> 5] = m;
-        __syncthreads();
-        uint32_t a = 0;
-        for (int k = 0; k < kStThreads / 32; ++k) a = max(a, warp_max[k]);
-        if (threadIdx.x == 0) {
-            const float af = __uint_as_float(a << 16);
-            const float sc = af > 0.0f ? __fdiv_rn(af, 448.0f) : 1.0f;
-            sm_inv = af > 0.0f ? __fdiv_rn(448.0f, af) : 1.0f;
-            *reinterpret_cast<float*>(en.chunk + ((uint64_t)p * H + h) * 4) = sc;
-        }
-        __syncthreads();
-        const float inv = sm_inv;
-        const uint64_t codes = en.chunk + f.scale_bytes + (uint64_t)p * n * H * D + (uint64_t)h * D + (uint64_t)w * 8;
-#pragma unroll
-        for (int u = 0; u < kHeadVec; ++u) {
-            const uint32_t i = i0 + u * step;
-            if (i < n) st_cs8(codes + (uint64_t)i * H * D, quant8(v[u], inv));
-        }
-        __syncthreads();                                   // warp_max / sm_inv are reused
+        if ((uint32_t)j.entries[e].n_tok == full_n)          // uniform across the CTA
+            store_head_segment<true>(f, e, p, h, warp_max, &sm_inv);
+        else
+            store_head_segment<false>(f, e, p, h, warp_max, &sm_inv);
     }
 }
 
