@@ -318,9 +318,13 @@ int kvs_get_choice(kvs_bw_report* out);
  * kvs_tune returns (the stream is synchronised).  KVS_F_MAX_CTAS(n) caps the
  * HOSTLINK candidate's grid (and becomes the host-link cap of that direction
  * if it wins); KVS_F_VALIDATE is honoured on the untimed runs; FORCE flags are
- * KVS_ERR_INVALID_ARG.  A call with no host-resident chunk changes nothing.
- * `out` (may be NULL) receives the rates in GB/s of host-chunk bytes (0 for a
- * candidate that cannot serve the call) and the choice.
+ * KVS_ERR_INVALID_ARG.  When the call holds device-resident chunks, those
+ * chunks alone are then timed with the LDG and the TMA kernel (TMA only for
+ * 16-byte aligned data), each chunk as a request of its own, and the faster
+ * kernel becomes the default for device chunks.  A call with no chunk of a
+ * class leaves that class's default unchanged.  `out` (may be NULL) receives
+ * the rates in GB/s of each class's bytes (0 for a candidate that cannot
+ * serve the call) and the choices.
  */
 #define KVS_DIR_RETRIEVE 0
 #define KVS_DIR_STORE    1
@@ -329,6 +333,10 @@ typedef struct kvs_tune_report {
     int64_t host_bytes;        /* bytes of host-resident chunks in the call             */
     int32_t chosen;            /* KVS_VARIANT_* now the default for this direction      */
     int32_t direction;         /* KVS_DIR_*                                             */
+    double  device_gbs[2];     /* device-resident chunks alone: [LDG, TMA] (0: not run)  */
+    int64_t device_bytes;      /* bytes of device-resident chunks in the call           */
+    int32_t chosen_kernel_device; /* KVS_KERNEL_* now the default for device chunks     */
+    int32_t reserved;
 } kvs_tune_report;
 int kvs_tune(const kvs_geometry* geom, const kvs_paged_cache* cache,
              const kvs_request* requests, int32_t num_requests,

@@ -1147,37 +1147,74 @@ int tune(DevState& st, const kvs_geometry* g, const kvs_paged_cache* cache, cons
                 host_bytes += (int64_t)2 * g->num_layers * reqs[r].chunks[j].num_tokens * (int64_t)pl.row_bytes;
     rep.host_bytes = host_bytes;
     rep.chosen = retrieve ? st.retrieve_host : st.store_host;
-    if (host_bytes == 0) {
-        if (out) *out = rep;
-        return KVS_OK;
-    }
+    rep.chosen_kernel_device = st.kernel_device;
     const uint32_t cap = flags & 0xFFFF0000u, base = flags & ~0xFFFF0000u;
-    const bool dma_ok = dma_pitch(st, pl, (uint64_t)g->block_size * pl.row_bytes) != 0;
-    const uint32_t cand[3] = {KVS_F_FORCE_HOSTLINK | cap, KVS_F_FORCE_HBMCOPY, KVS_F_FORCE_DMA};
-    for (int v = 0; v < 3; ++v) {
-        if (v == 2 && !dma_ok) continue;
-        rc = copy_call(g, cache, reqs, nreq, (void*)s, base | cand[v], retrieve);   // untimed (validated if asked)
-        if (rc) return rc;
+    auto timed = [&](const kvs_request* rq, int32_t n, uint32_t fl, int64_t bytes, double* gbs) -> int {
+        int rc2 = copy_call(g, cache, rq, n, (void*)s, base | fl, retrieve);      // untimed (validated if asked)
+        if (rc2) return rc2;
         double best = 0;
-        rc = time_best(s, reps, &best, [&]() -> int {
-            return copy_call(g, cache, reqs, nreq, (void*)s, (base & ~KVS_F_VALIDATE) | cand[v], retrieve);
+        rc2 = time_best(s, reps, &best, [&]() -> int {
+            return copy_call(g, cache, rq, n, (void*)s, (base & ~KVS_F_VALIDATE) | fl, retrieve);
         });
+        if (rc2) return rc2;
+        *gbs = (double)bytes / (best * 1e6);
+        return KVS_OK;
+    };
+    if (host_bytes > 0) {
+        const bool dma_ok = dma_pitch(st, pl, (uint64_t)g->block_size * pl.row_bytes) != 0;
+        const uint32_t cand[3] = {KVS_F_FORCE_HOSTLINK | cap, KVS_F_FORCE_HBMCOPY, KVS_F_FORCE_DMA};
+        for (int v = 0; v < 3; ++v) {
+            if (v == 2 && !dma_ok) continue;
+            rc = timed(reqs, nreq, cand[v], host_bytes, &rep.gbs[v]);
+            if (rc) return rc;
+        }
+        int v = 0;
+        for (int k = 1; k < 3; ++k)
+            if (rep.gbs[k] > rep.gbs[v]) v = k;
+        const int chosen = v == 0 ? KVS_VARIANT_HOSTLINK : v == 1 ? KVS_VARIANT_HBMCOPY : KVS_VARIANT_DMA;
+        if (retrieve) {
+            st.retrieve_host = chosen;
+            if (chosen == KVS_VARIANT_HOSTLINK && cap) st.hostlink_ctas = (int)KVS_F_GET_MAX_CTAS(flags);
+        } else {
+            st.store_host = chosen;
+            if (chosen == KVS_VARIANT_HOSTLINK && cap) st.store_ctas = (int)KVS_F_GET_MAX_CTAS(flags);
+        }
+        rep.chosen = chosen;
+    }
+    // Device-resident chunks: the LDG and TMA kernels on those chunks alone.  Each
+    // becomes a one-chunk request starting at its own first token (a multiple of
+    // chunk_tokens: every chunk before it is full), with the request's block table.
+    std::vector<kvs_chunk> dch;
+    std::vector<kvs_request> dreq;
+    int64_t device_bytes = 0;
+    for (int32_t r = 0; r < nreq; ++r)
+        for (int32_t j = 0; j < reqs[r].num_chunks; ++j)
+            if (reqs[r].chunks[j].residency == KVS_SRC_DEVICE) dch.push_back(reqs[r].chunks[j]);
+    dreq.reserve(dch.size());
+    for (int32_t r = 0, k = 0; r < nreq; ++r) {
+        int64_t s0 = reqs[r].first_token;
+        for (int32_t j = 0; j < reqs[r].num_chunks; ++j) {
+            const kvs_chunk& c = reqs[r].chunks[j];
+            if (c.residency == KVS_SRC_DEVICE) {
+                dreq.push_back({s0, c.num_tokens, &dch[k++], 1, reqs[r].block_table_len, reqs[r].block_table});
+                device_bytes += (int64_t)2 * g->num_layers * c.num_tokens * (int64_t)pl.row_bytes;
+            }
+            s0 += c.num_tokens;
+        }
+    }
+    rep.device_bytes = device_bytes;
+    if (device_bytes > 0) {
+        rc = timed(dreq.data(), (int32_t)dreq.size(), KVS_F_FORCE_LDG, device_bytes, &rep.device_gbs[0]);
         if (rc) return rc;
-        rep.gbs[v] = (double)host_bytes / (best * 1e6);
+        if (vec_bytes_for(pl.addr_or) == 16) {      // TMA needs 16-byte aligned planes and rows
+            rc = timed(dreq.data(), (int32_t)dreq.size(), KVS_F_FORCE_TMA, device_bytes, &rep.device_gbs[1]);
+            if (rc == KVS_ERR_UNSUPPORTED) { rep.device_gbs[1] = 0; rc = KVS_OK; t_error.clear(); }
+            if (rc) return rc;
+        }
+        st.kernel_device = rep.device_gbs[1] > rep.device_gbs[0] ? KVS_KERNEL_TMA : KVS_KERNEL_LDG;
+        rep.chosen_kernel_device = st.kernel_device;
     }
     KVS_CUDA(cudaStreamSynchronize(s));
-    int v = 0;
-    for (int k = 1; k < 3; ++k)
-        if (rep.gbs[k] > rep.gbs[v]) v = k;
-    const int chosen = v == 0 ? KVS_VARIANT_HOSTLINK : v == 1 ? KVS_VARIANT_HBMCOPY : KVS_VARIANT_DMA;
-    if (retrieve) {
-        st.retrieve_host = chosen;
-        if (chosen == KVS_VARIANT_HOSTLINK && cap) st.hostlink_ctas = (int)KVS_F_GET_MAX_CTAS(flags);
-    } else {
-        st.store_host = chosen;
-        if (chosen == KVS_VARIANT_HOSTLINK && cap) st.store_ctas = (int)KVS_F_GET_MAX_CTAS(flags);
-    }
-    rep.chosen = chosen;
     if (out) *out = rep;
     return KVS_OK;
 }

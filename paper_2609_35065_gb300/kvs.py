@@ -128,7 +128,8 @@ class kvs_bw_report(ctypes.Structure):
 
 class kvs_tune_report(ctypes.Structure):
     _fields_ = [("gbs", ctypes.c_double * 3), ("host_bytes", ctypes.c_int64), ("chosen", ctypes.c_int32),
-                ("direction", ctypes.c_int32)]
+                ("direction", ctypes.c_int32), ("device_gbs", ctypes.c_double * 2), ("device_bytes", ctypes.c_int64),
+                ("chosen_kernel_device", ctypes.c_int32), ("reserved", ctypes.c_int32)]
 
 
 class kvs_tier_config(ctypes.Structure):
@@ -416,7 +417,9 @@ def kvs_tune(geom, planes, num_blocks, requests, stream=None, flags: int = 0,
     rep = kvs_tune_report()
     _check(lib().kvs_tune(ctypes.byref(g), ctypes.byref(m.cache), m.reqs, m.n, _stream(stream),
                           ctypes.c_uint32(flags), int(direction), int(reps), ctypes.byref(rep)))
-    return {"gbs": list(rep.gbs), "host_bytes": rep.host_bytes, "chosen": rep.chosen, "direction": rep.direction}
+    return {"gbs": list(rep.gbs), "host_bytes": rep.host_bytes, "chosen": rep.chosen, "direction": rep.direction,
+            "device_gbs": list(rep.device_gbs), "device_bytes": rep.device_bytes,
+            "chosen_kernel_device": rep.chosen_kernel_device}
 
 
 def kvs_get_choice() -> dict:

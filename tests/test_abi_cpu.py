@@ -34,7 +34,7 @@ def test_struct_layouts_match_header():
     assert ctypes.sizeof(kvs.kvs_request) == 40
     assert ctypes.sizeof(kvs.kvs_paged_cache) == 16
     assert ctypes.sizeof(kvs.kvs_bw_report) == 5 * 8 + 6 * 8 + 6 * 4 + 8 + 2 * 8
-    assert ctypes.sizeof(kvs.kvs_tune_report) == 3 * 8 + 8 + 2 * 4
+    assert ctypes.sizeof(kvs.kvs_tune_report) == 3 * 8 + 8 + 2 * 4 + 2 * 8 + 8 + 2 * 4
 
 
 class _Arena:

@@ -150,13 +150,43 @@ def test_tune_argument_checks():
         with pytest.raises(kvs.KvsError) as ei:
             kvs.kvs_tune(w.geom, buf.plane_ptrs, w.num_blocks, buf.requests, None, flags, direction, reps)
         assert ei.value.code == kvs.KVS_ERR_INVALID_ARG
-    # device-resident chunks only: nothing to choose, nothing changes
+    # device-resident chunks only: the host-chunk choice is left alone
     w2 = synth.tiny()
     w2.requests[0].residency = "device"
     b2 = buffers.allocate(w2)
     before = kvs.kvs_get_choice()["chosen_retrieve_host"]
     rep = kvs.kvs_tune(w2.geom, b2.plane_ptrs, w2.num_blocks, b2.requests, None, 0, 0, 1)
-    assert rep["host_bytes"] == 0 and rep["chosen"] == before
+    assert rep["host_bytes"] == 0 and rep["chosen"] == before and rep["gbs"] == [0, 0, 0]
+
+
+@pytest.mark.parametrize("direction", [kvs.KVS_DIR_RETRIEVE, kvs.KVS_DIR_STORE], ids=["retrieve", "store"])
+def test_tune_chooses_the_device_kernel_by_measurement(direction):
+    """Mixed residency (the sweep's shape, scaled down): host chunks are tuned over the host
+    variants, the device chunks alone over LDG and TMA; the faster kernel becomes the
+    device default, and a default call afterwards equals the oracle."""
+    w = synth.custom(4, 8, 128, 16, 256, 600, [2048, 2048, 1536, 1024], [1536, 1024, 1536, 768], seed=4,
+                     dist="normal", residency=["host", "device", "device", "host"],
+                     store_tokens=[256, 512, 0, 256])
+    buf = buffers.allocate(w, store=True, store_residency="device")
+    g = w.geom
+    reqs = buf.requests if direction == kvs.KVS_DIR_RETRIEVE else buf.store_requests
+    if direction == kvs.KVS_DIR_STORE:
+        kvs.kvs_retrieve(g, buf.plane_ptrs, w.num_blocks, buf.requests, None, kvs.KVS_F_VALIDATE)
+    rep = kvs.kvs_tune(g, buf.plane_ptrs, w.num_blocks, reqs, None, 0, direction, reps=2)
+    assert rep["device_bytes"] > 0 and min(rep["device_gbs"]) > 0, rep
+    want = kvs.KVS_KERNEL_TMA if rep["device_gbs"][1] > rep["device_gbs"][0] else kvs.KVS_KERNEL_LDG
+    assert rep["chosen_kernel_device"] == want == kvs.kvs_get_choice()["chosen_kernel_device"]
+    if direction == kvs.KVS_DIR_RETRIEVE:
+        _sentinel(buf)
+        kvs.kvs_retrieve(g, buf.plane_ptrs, w.num_blocks, reqs, None, kvs.KVS_F_VALIDATE)
+        gc.check_retrieve(buf)
+    else:
+        for mine in buf.store_chunks:
+            for t in mine:
+                t.fill_(0)
+        kvs.kvs_store(g, buf.plane_ptrs, w.num_blocks, reqs, None, kvs.KVS_F_VALIDATE)
+        gc.check_store(buf)
+    kvs.kvs_shutdown()
 
 
 @pytest.mark.parametrize("cap", [0, 3, 12], ids=["default_grid", "3_ctas", "12_ctas"])
