@@ -1361,43 +1361,47 @@ int kvs_enqueue_error_read(void* cuda_stream, int32_t* host_word) {
 const char* kvs_last_error(void) { return t_error.c_str(); }
 
 int kvs_shutdown(void) {
-    std::lock_guard<std::mutex> lk(g_mu);
-    int prev = 0;
-    cudaGetDevice(&prev);
-    for (auto& st : g_dev) {
-        if (!st.ready) continue;
-        cudaSetDevice(st.device);
-        cudaDeviceSynchronize();
-        for (auto& sl : st.up) {
-            if (sl.host) cudaFreeHost(sl.host);
-            if (sl.dev) cudaFree(sl.dev);
-            if (sl.done) cudaEventDestroy(sl.done);
-            if (sl.uploaded) cudaEventDestroy(sl.uploaded);
-        }
-        if (st.upload_stream) cudaStreamDestroy(st.upload_stream);
-        for (int k = 0; k < kRingSlots; ++k) {
-            cudaEventDestroy(st.ring_filled[k]);
-            cudaEventDestroy(st.ring_free[k]);
-        }
-        cudaEventDestroy(st.ev_fork);
-        cudaEventDestroy(st.ev_join);
-        cudaEventDestroy(st.ev_aux_fork);
-        cudaEventDestroy(st.ev_aux_join);
-        if (st.aux_stream) cudaStreamDestroy(st.aux_stream);
-        for (auto& sg : st.sig) {
-            if (sg.mem) cudaFree(sg.mem);
-            if (sg.done) cudaEventDestroy(sg.done);
-        }
-        if (st.signal_stream) cudaStreamDestroy(st.signal_stream);
-        if (st.ring) cudaFree(st.ring);
-        if (st.copy_stream) cudaStreamDestroy(st.copy_stream);
-        if (st.err) cudaFree(st.err);
-        if (st.err_host) cudaFreeHost(st.err_host);
-        st = DevState{};
+    // The allocation-free entry point takes its own lock and then this one (for
+    // the host-link cap), so its address is forgotten after this lock is released.
+    {
+        std::lock_guard<std::mutex> lk(g_mu);
+        int prev = 0;
+        cudaGetDevice(&prev);
+        for (auto& st : g_dev) {
+            if (!st.ready) continue;
+            cudaSetDevice(st.device);
+            cudaDeviceSynchronize();
+            for (auto& sl : st.up) {
+                if (sl.host) cudaFreeHost(sl.host);
+                if (sl.dev) cudaFree(sl.dev);
+                if (sl.done) cudaEventDestroy(sl.done);
+                if (sl.uploaded) cudaEventDestroy(sl.uploaded);
+            }
+            if (st.upload_stream) cudaStreamDestroy(st.upload_stream);
+            for (int k = 0; k < kRingSlots; ++k) {
+                cudaEventDestroy(st.ring_filled[k]);
+                cudaEventDestroy(st.ring_free[k]);
+            }
+            cudaEventDestroy(st.ev_fork);
+            cudaEventDestroy(st.ev_join);
+            cudaEventDestroy(st.ev_aux_fork);
+            cudaEventDestroy(st.ev_aux_join);
+            if (st.aux_stream) cudaStreamDestroy(st.aux_stream);
+            for (auto& sg : st.sig) {
+                if (sg.mem) cudaFree(sg.mem);
+                if (sg.done) cudaEventDestroy(sg.done);
+            }
+            if (st.signal_stream) cudaStreamDestroy(st.signal_stream);
+            if (st.ring) cudaFree(st.ring);
+            if (st.copy_stream) cudaStreamDestroy(st.copy_stream);
+            if (st.err) cudaFree(st.err);
+            if (st.err_host) cudaFreeHost(st.err_host);
+            st = DevState{};
     }
     g_dev.clear();
-    noalloc_forget_devices();
     cudaSetDevice(prev);
+    }
+    noalloc_forget_devices();
     return KVS_OK;
 }
 
