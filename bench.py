@@ -1227,10 +1227,16 @@ def run_tempokv(args):
     rates = {"pcie_context_16.8": 16.8}
     if measured:
         rates["gb300_measured"] = round(measured, 2)
+    # fp8 chunks (E4M3 codes + one binary32 scale per layer, K/V and head per 256-token chunk):
+    # 64 KiB + 8 bytes per token at the 8B geometry, moved at the same link rate (the fp8
+    # kernel holds 99% of the link, bench.py --fp8)
+    scenarios = {name: (gbs, 128 * 1024) for name, gbs in rates.items()}
+    if measured:
+        scenarios["gb300_measured_fp8_chunks"] = (round(measured, 2), 64 * 1024 + 2 * 32 * 8 * 4 // 256)
     out = {}
     t0 = _time.perf_counter()
-    for name, gbs in rates.items():
-        cal = tempokv.Calibration(retrieval_gbs=gbs)
+    for name, (gbs, per_tok) in scenarios.items():
+        cal = tempokv.Calibration(retrieval_gbs=gbs, kv_bytes_per_token=per_tok)
         for ratio in (0.5, 0.75, 1.0):
             res = tempokv.simulate(tempokv.workload(ratio, cal=cal), cal)
             out[f"{name}/ratio{int(ratio * 100)}"] = {
@@ -1242,7 +1248,8 @@ def run_tempokv(args):
             "unit": "s / tok/s / GiB.s per request", "config": {
                 "workload": "12 synthetic documents, 16,078-67,744 tokens, arrivals every 0.5 s, <= 128 output tokens",
                 "fast_tier": "100 GiB, protected budget 50 GiB, 11 GiB/s staging, FCFS <= 4 active",
-                "retrieval_gbs": rates}, "results": out,
+                "retrieval_gbs": rates,
+                "kv_bytes_per_token": {k: v[1] for k, v in scenarios.items()}}, "results": out,
             "model_seconds": round(_time.perf_counter() - t0, 2)}
     print(json.dumps(line), flush=True)
     return 0

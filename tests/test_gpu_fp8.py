@@ -162,3 +162,27 @@ def test_fp8_store_two_pass_for_large_heads(residency):
     _store(buf)
     torch.cuda.synchronize()
     gc.check_store_fp8(buf)
+
+
+def test_fp8_qwen14b_shape_retrieve_and_suffix_store():
+    """48 layers (192 KiB of BF16 per token), two requests of 12,288 matched tokens
+    (48 chunks each, 2.25 GiB of fp8 chunks in pinned host memory) dequantised, then the
+    computed 4096-token suffix of each stored back into fp8 chunks; every element of all
+    96 planes and every byte of the stored chunks against the oracle."""
+    w = synth.qwen14b(requests=2, num_blocks=2048, shared_frac=0.0)
+    assert w.notes["shared_blocks"] == 0
+    buf = buffers.allocate_fp8(w, store=True)
+    s = torch.cuda.Stream()
+    kvs.kvs_retrieve_fp8(w.geom, buf.plane_ptrs, w.num_blocks, buf.requests, s, 0)
+    s.synchronize()
+    assert kvs.kvs_check_errors(s) == kvs.KVS_OK
+    gc.check_retrieve_fp8(buf)
+    # the suffix blocks hold computed KV: seeded normal values in every plane
+    gen = torch.Generator(device="cuda").manual_seed(14)
+    for p in range(buf.planes.shape[0]):
+        synth.fill_values(buf.planes[p], "normal", gen)
+    torch.cuda.synchronize()
+    kvs.kvs_store_fp8(w.geom, buf.plane_ptrs, w.num_blocks, buf.store_requests, s, 0)
+    s.synchronize()
+    assert kvs.kvs_check_errors(s) == kvs.KVS_OK
+    gc.check_store_fp8(buf)
