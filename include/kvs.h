@@ -266,6 +266,19 @@ int kvs_store_fp8(const kvs_geometry* geom, const kvs_paged_cache* cache,
                   const kvs_request* requests, int32_t num_requests,
                   void* cuda_stream, uint32_t flags);
 
+/* Layer-wise forms of the two fp8 calls, with the semantics of kvs_retrieve_layers
+ * / kvs_store_layers (the model can start on layer group k once layer_events[k]
+ * fires; group k of a store waits on ready_events[k]): one launch per layer
+ * group and source class, on cuda_stream.  KVS_F_LAYER_SIGNAL is not accepted. */
+int kvs_retrieve_fp8_layers(const kvs_geometry* geom, const kvs_paged_cache* cache,
+                            const kvs_request* requests, int32_t num_requests,
+                            int32_t layers_per_step, void* const* layer_events,
+                            void* cuda_stream, uint32_t flags);
+int kvs_store_fp8_layers(const kvs_geometry* geom, const kvs_paged_cache* cache,
+                         const kvs_request* requests, int32_t num_requests,
+                         int32_t layers_per_step, void* const* ready_events,
+                         void* const* layer_events, void* cuda_stream, uint32_t flags);
+
 /* Bandwidths measured by kvs_query_bw, in GB/s (1e9 bytes per second). */
 typedef struct kvs_bw_report {
     double  hbm_copy_gbs;          /* device->device copy kernel, read + write bytes      */

@@ -873,8 +873,11 @@ int copy_call(const kvs_geometry* g, const kvs_paged_cache* cache, const kvs_req
 // same stream.  A physical block named by two requests is refused: the
 // quantised copies of a shared block differ with each chunk's scales, so no
 // single writer would be the right one.
+// layers_per_step > 0: layer groups in layer order, each preceded by a wait on
+// ready_events[k] and followed by a record of layer_events[k] (either if given).
 int fp8_call(const kvs_geometry* g, const kvs_paged_cache* cache, const kvs_request* reqs,
-             int32_t nreq, void* stream, uint32_t flags, bool retrieve) {
+             int32_t nreq, void* stream, uint32_t flags, bool retrieve, int32_t layers_per_step = 0,
+             void* const* layer_events = nullptr, void* const* ready_events = nullptr) {
     const uint32_t allowed = KVS_F_VALIDATE | KVS_F_FORCE_HOSTLINK | KVS_F_FORCE_LDG | 0xFFFF0000u;
     if (flags & ~allowed)
         return fail(KVS_ERR_UNSUPPORTED, "fp8 calls take only KVS_F_VALIDATE, KVS_F_FORCE_HOSTLINK, "
@@ -897,7 +900,13 @@ int fp8_call(const kvs_geometry* g, const kvs_paged_cache* cache, const kvs_requ
         rc = check_overlaps(g, cache, reqs, nreq, retrieve, true);
         if (rc) return rc;
     }
-    if (pl.num_device + pl.num_host == 0) return KVS_OK;
+    if (pl.num_device + pl.num_host == 0) {
+        // nothing to copy: the layer events still mark "ready" in stream order
+        if (layers_per_step > 0 && layer_events)
+            for (int k = 0; k < (g->num_layers + layers_per_step - 1) / layers_per_step; ++k)
+                if (layer_events[k]) KVS_CUDA(cudaEventRecord((cudaEvent_t)layer_events[k], (cudaStream_t)stream));
+        return KVS_OK;
+    }
     DevState* stp = nullptr;
     rc = get_state(&stp);
     if (rc) return rc;
@@ -917,9 +926,9 @@ int fp8_call(const kvs_geometry* g, const kvs_paged_cache* cache, const kvs_requ
     SlotGuard guard{u.slot, s};
     const int cap = (int)KVS_F_GET_MAX_CTAS(flags);
     const uint32_t hd = (uint32_t)(g->num_kv_heads * g->head_dim);
-    auto fjob = [&](uint32_t first, uint32_t count) {
+    auto fjob = [&](uint32_t first, uint32_t count, uint32_t p0, uint32_t np) {
         Fp8Job f{};
-        f.job = make_job(st, g, cache, pl, u, first, count, retrieve ? MODE_RETRIEVE : MODE_STORE);
+        f.job = make_job(st, g, cache, pl, u, first, count, retrieve ? MODE_RETRIEVE : MODE_STORE, p0, np);
         const uint64_t run_codes = (uint64_t)g->block_size * hd;
         f.job.pieces_per_run = (uint32_t)((run_codes + kFp8PieceCodes - 1) / kFp8PieceCodes);
         f.job.num_pieces = (uint64_t)count * f.job.num_planes * f.job.blocks_per_chunk * f.job.pieces_per_run;
@@ -937,23 +946,33 @@ int fp8_call(const kvs_geometry* g, const kvs_paged_cache* cache, const kvs_requ
         ++g_launches;
         return KVS_OK;
     };
-    if (pl.num_host) {
-        const Fp8Job f = fjob(pl.num_device, pl.num_host);
-        if (f.job.num_pieces >= (1ull << 31)) return fail(KVS_ERR_INVALID_ARG, "call too large: split it");
-        // Retrieval: a CTA keeps up to 32 KiB of codes in flight, half a link-kernel
-        // CTA's bytes, so it takes twice the link kernel's grid.  Store-back: one CTA
-        // per (chunk, plane) over the whole GPU (its two passes are not pipelined
-        // across segments, so a capped grid would be latency-bound).
-        const int grid = cap ? cap : (retrieve ? 2 * st.hostlink_ctas : 0);
-        rc = run(f, grid);
-        if (rc) return rc;
-    }
-    if (pl.num_device) {
-        const Fp8Job f = fjob(0, pl.num_device);
-        if (f.job.num_pieces >= (1ull << 31)) return fail(KVS_ERR_INVALID_ARG, "call too large: split it");
-        // HBM chunks: uncapped retrievals run one CTA per piece
-        rc = run(f, cap ? cap : (retrieve ? kFp8PerPiece : 0));
-        if (rc) return rc;
+    const int L = g->num_layers;
+    const int lps = layers_per_step > 0 ? std::min(layers_per_step, L) : L;
+    const int groups = (L + lps - 1) / lps;
+    for (int k = 0; k < groups; ++k) {
+        const uint32_t p0 = (uint32_t)(2 * k * lps);
+        const uint32_t np = (uint32_t)(2 * (std::min(L, (k + 1) * lps) - k * lps));
+        if (ready_events && ready_events[k])
+            KVS_CUDA(cudaStreamWaitEvent(s, (cudaEvent_t)ready_events[k], 0));
+        if (pl.num_host) {
+            const Fp8Job f = fjob(pl.num_device, pl.num_host, p0, np);
+            if (f.job.num_pieces >= (1ull << 31)) return fail(KVS_ERR_INVALID_ARG, "call too large: split it");
+            // Retrieval: a CTA keeps up to 32 KiB of codes in flight, half a link-kernel
+            // CTA's bytes, so it takes twice the link kernel's grid.  Store-back: one CTA
+            // per (chunk, plane, head) over the whole GPU.
+            const int grid = cap ? cap : (retrieve ? 2 * st.hostlink_ctas : 0);
+            rc = run(f, grid);
+            if (rc) return rc;
+        }
+        if (pl.num_device) {
+            const Fp8Job f = fjob(0, pl.num_device, p0, np);
+            if (f.job.num_pieces >= (1ull << 31)) return fail(KVS_ERR_INVALID_ARG, "call too large: split it");
+            // HBM chunks: uncapped retrievals run one CTA per piece
+            rc = run(f, cap ? cap : (retrieve ? kFp8PerPiece : 0));
+            if (rc) return rc;
+        }
+        if (layers_per_step > 0 && layer_events && layer_events[k])
+            KVS_CUDA(cudaEventRecord((cudaEvent_t)layer_events[k], s));
     }
     if (flags & KVS_F_VALIDATE) {
         KVS_CUDA(cudaEventRecord(u.slot->done, s));
@@ -1272,6 +1291,25 @@ int kvs_store_fp8(const kvs_geometry* geom, const kvs_paged_cache* cache, const 
     std::lock_guard<std::mutex> lk(g_mu);
     t_error.clear();
     return fp8_call(geom, cache, requests, num_requests, cuda_stream, flags, false);
+}
+
+int kvs_retrieve_fp8_layers(const kvs_geometry* geom, const kvs_paged_cache* cache, const kvs_request* requests,
+                            int32_t num_requests, int32_t layers_per_step, void* const* layer_events,
+                            void* cuda_stream, uint32_t flags) {
+    std::lock_guard<std::mutex> lk(g_mu);
+    t_error.clear();
+    if (layers_per_step <= 0) return fail(KVS_ERR_INVALID_ARG, "layers_per_step must be positive");
+    return fp8_call(geom, cache, requests, num_requests, cuda_stream, flags, true, layers_per_step, layer_events);
+}
+
+int kvs_store_fp8_layers(const kvs_geometry* geom, const kvs_paged_cache* cache, const kvs_request* requests,
+                         int32_t num_requests, int32_t layers_per_step, void* const* ready_events,
+                         void* const* layer_events, void* cuda_stream, uint32_t flags) {
+    std::lock_guard<std::mutex> lk(g_mu);
+    t_error.clear();
+    if (layers_per_step <= 0) return fail(KVS_ERR_INVALID_ARG, "layers_per_step must be positive");
+    return fp8_call(geom, cache, requests, num_requests, cuda_stream, flags, false, layers_per_step, layer_events,
+                    ready_events);
 }
 
 int kvs_retrieve_layers(const kvs_geometry* geom, const kvs_paged_cache* cache, const kvs_request* requests,

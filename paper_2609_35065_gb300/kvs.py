@@ -65,7 +65,7 @@ EXPORTED = ("kvs_retrieve", "kvs_store", "kvs_query_bw", "kvs_get_choice", "kvs_
             "kvs_enqueue_error_read",
             "kvs_last_error", "kvs_shutdown", "kvs_version", "kvs_selftest_wait_timeout",
             "kvs_stat_launches", "kvs_retrieve_noalloc", "kvs_retrieve_layers", "kvs_store_layers",
-            "kvs_retrieve_fp8", "kvs_store_fp8", "kvs_tune",
+            "kvs_retrieve_fp8", "kvs_store_fp8", "kvs_retrieve_fp8_layers", "kvs_store_fp8_layers", "kvs_tune",
             "kvs_tier_create", "kvs_tier_destroy", "kvs_tier_commit", "kvs_tier_staged",
             "kvs_tier_begin_retrieval", "kvs_tier_end_retrieval", "kvs_tier_cancel", "kvs_tier_ordinary",
             "kvs_tier_claim_state", "kvs_tier_object", "kvs_tier_stats_get", "kvs_tier_slot")
@@ -184,6 +184,10 @@ def lib():
                                            ctypes.POINTER(kvs_request), ctypes.c_int32, ctypes.c_int32,
                                            EVP, EVP, P, ctypes.c_uint32]
             L.kvs_store_layers.restype = ctypes.c_int
+            L.kvs_retrieve_fp8_layers.argtypes = L.kvs_retrieve_layers.argtypes
+            L.kvs_retrieve_fp8_layers.restype = ctypes.c_int
+            L.kvs_store_fp8_layers.argtypes = L.kvs_store_layers.argtypes
+            L.kvs_store_fp8_layers.restype = ctypes.c_int
             U64P, I64P, I32P = (ctypes.POINTER(ctypes.c_uint64), ctypes.POINTER(ctypes.c_int64),
                                 ctypes.POINTER(ctypes.c_int32))
             tier_sigs = {
@@ -484,6 +488,27 @@ def kvs_store_fp8(geom, planes, num_blocks, requests, stream=None, flags: int = 
     m = _Marshalled(planes, num_blocks, requests)
     return _check(lib().kvs_store_fp8(ctypes.byref(g), ctypes.byref(m.cache), m.reqs, m.n,
                                       _stream(stream), ctypes.c_uint32(flags)))
+
+
+def kvs_retrieve_fp8_layers(geom, planes, num_blocks, requests, layers_per_step, layer_events=None,
+                            stream=None, flags: int = 0) -> int:
+    """Layer-wise :func:`kvs_retrieve_fp8`; ``layer_events[k]`` is recorded after group k."""
+    g = _geometry(geom)
+    m = _Marshalled(planes, num_blocks, requests)
+    keep, ev = _events(layer_events, stream)
+    return _check(lib().kvs_retrieve_fp8_layers(ctypes.byref(g), ctypes.byref(m.cache), m.reqs, m.n,
+                                                int(layers_per_step), ev, _stream(stream), ctypes.c_uint32(flags)))
+
+
+def kvs_store_fp8_layers(geom, planes, num_blocks, requests, layers_per_step, layer_events=None,
+                         stream=None, flags: int = 0, ready_events=None) -> int:
+    """Layer-wise :func:`kvs_store_fp8`: group k waits on ``ready_events[k]``."""
+    g = _geometry(geom)
+    m = _Marshalled(planes, num_blocks, requests)
+    keep_r, rev = _wait_events(ready_events)
+    keep, ev = _events(layer_events, stream)
+    return _check(lib().kvs_store_fp8_layers(ctypes.byref(g), ctypes.byref(m.cache), m.reqs, m.n,
+                                             int(layers_per_step), rev, ev, _stream(stream), ctypes.c_uint32(flags)))
 
 
 # ---- fast tier ------------------------------------------------------------

@@ -186,3 +186,70 @@ def test_fp8_qwen14b_shape_retrieve_and_suffix_store():
     s.synchronize()
     assert kvs.kvs_check_errors(s) == kvs.KVS_OK
     gc.check_store_fp8(buf)
+
+
+@pytest.mark.parametrize("lps", [1, 3])
+@pytest.mark.parametrize("residency", ["host", "mixed"])
+def test_fp8_layer_groups_are_ready_when_their_event_fires(lps, residency):
+    """Layer-wise fp8 retrieval: a consumer stream that waits on layer_events[k] sees
+    group k dequantised exactly as the oracle's, whatever later groups are doing."""
+    res = ["host", "device", "host"] if residency == "mixed" else residency
+    w = synth.custom(5, 8, 128, 16, 256, 200, [1024, 768, 1280], [1024, 768, 1024], seed=8, residency=res)
+    g = w.geom
+    buf = buffers.allocate_fp8(w)
+    groups = -(-g.layers // lps)
+    events = [torch.cuda.Event() for _ in range(groups)]
+    copier, consumer = torch.cuda.Stream(), torch.cuda.Stream()
+    kvs.kvs_retrieve_fp8_layers(g, buf.plane_ptrs, w.num_blocks, buf.requests, lps, events, copier, 0)
+    snaps = []
+    for k, ev in enumerate(events):
+        consumer.wait_event(ev)
+        p0, p1 = 2 * k * lps, 2 * min(g.layers, (k + 1) * lps)
+        with torch.cuda.stream(consumer):
+            snaps.append((p0, p1, buf.planes[p0:p1].clone()))
+    torch.cuda.synchronize()
+    assert kvs.kvs_check_errors(None) == kvs.KVS_OK
+    chunks_np = [[gc._np(t) for t in mine] for mine in buf.chunks]
+    for p0, p1, snap in snaps:
+        for p in range(p0, p1):
+            want = gc.expected_plane_fp8(buf, p, chunks_np)
+            assert np.array_equal(snap[p - p0].cpu().numpy().view(np.uint16), want), (lps, p)
+    gc.check_retrieve_fp8(buf, chunks_np=chunks_np)
+
+
+def test_fp8_layerwise_store_waits_for_ready_events():
+    """Layer-wise fp8 store-back: a producer rewrites each layer group's planes after a
+    delay and then records its ready event; the stored chunks equal the oracle's store of
+    the rewritten planes."""
+    w = synth.custom(4, 8, 128, 16, 256, 200, [1024, 768], [0, 0], seed=12, store_tokens=[1024, 768])
+    g = w.geom
+    buf = buffers.allocate_fp8(w, store=True)
+    lps = 2
+    groups = -(-g.layers // lps)
+    ready = [torch.cuda.Event() for _ in range(groups)]
+    done = [torch.cuda.Event() for _ in range(groups)]
+    producer, copier = torch.cuda.Stream(), torch.cuda.Stream()
+    gen = torch.Generator(device="cuda").manual_seed(12)
+    with torch.cuda.stream(producer):
+        for k in range(groups):
+            torch.cuda._sleep(20_000_000)
+            for p in range(2 * k * lps, 2 * min(g.layers, (k + 1) * lps)):
+                synth.fill_values(buf.planes[p], "normal", gen)
+            ready[k].record(producer)
+    kvs.kvs_store_fp8_layers(g, buf.plane_ptrs, w.num_blocks, buf.store_requests, lps, done, copier, 0,
+                             ready_events=ready)
+    torch.cuda.synchronize()
+    assert kvs.kvs_check_errors(None) == kvs.KVS_OK
+    gc.check_store_fp8(buf)
+
+
+def test_fp8_layerwise_argument_checks():
+    w = synth.custom(2, 2, 32, 16, 32, 8, [64], [32])
+    buf = buffers.allocate_fp8(w)
+    for fn in (kvs.kvs_retrieve_fp8_layers, kvs.kvs_store_fp8_layers):
+        with pytest.raises(kvs.KvsError) as ei:
+            fn(w.geom, buf.plane_ptrs, w.num_blocks, buf.requests, 0)
+        assert ei.value.code == kvs.KVS_ERR_INVALID_ARG
+        with pytest.raises(kvs.KvsError) as ei:
+            fn(w.geom, buf.plane_ptrs, w.num_blocks, buf.requests, 1, None, None, kvs.KVS_F_LAYER_SIGNAL)
+        assert ei.value.code == kvs.KVS_ERR_UNSUPPORTED
