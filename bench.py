@@ -1056,6 +1056,8 @@ def run_layerwise(args):
     for r in w.requests:                  # the computed suffix is stored back into chunks
         r.store_tokens = r.prompt_tokens - r.matched_tokens
     buf = buffers.allocate(w, store=True)
+    # the same prefix and suffix as fp8 chunks (E4M3 + per-head scales), into the same planes
+    fb = buffers.allocate_fp8(w, store=True, with_planes=False)
     suffix = sum(r.prompt_tokens - r.matched_tokens for r in w.requests)
     # per-layer prefill work of the suffix: q/k/v + o + gated MLP widths of Llama-3-8B
     M, K, N = suffix, 4096, (4096 + 2 * 1024) + 4096 + 3 * 14336
@@ -1067,8 +1069,29 @@ def run_layerwise(args):
     def ev():
         return torch.cuda.Event(enable_timing=True)
 
+    def copies(fp8):
+        """The four copy calls, BF16 or fp8 chunks."""
+        if fp8:
+            return (lambda: kvs.kvs_retrieve_fp8(g, buf.plane_ptrs, w.num_blocks, fb.requests, side, 0),
+                    lambda: kvs.kvs_store_fp8(g, buf.plane_ptrs, w.num_blocks, fb.store_requests, side, 0),
+                    lambda lps, evs, fl: kvs.kvs_retrieve_fp8_layers(g, buf.plane_ptrs, w.num_blocks, fb.requests,
+                                                                     lps, evs, side, fl),
+                    lambda lps, fl, ready: kvs.kvs_store_fp8_layers(g, buf.plane_ptrs, w.num_blocks,
+                                                                    fb.store_requests, lps, None, side, fl,
+                                                                    ready_events=ready))
+        return (lambda: kvs.kvs_retrieve(g, buf.plane_ptrs, w.num_blocks, buf.requests, side, 0),
+                lambda: kvs.kvs_store(g, buf.plane_ptrs, w.num_blocks, buf.store_requests, side, 0),
+                lambda lps, evs, fl: kvs.kvs_retrieve_layers(g, buf.plane_ptrs, w.num_blocks, buf.requests,
+                                                             lps, evs, side, fl),
+                lambda lps, fl, ready: kvs.kvs_store_layers(g, buf.plane_ptrs, w.num_blocks, buf.store_requests,
+                                                            lps, None, side, fl, ready_events=ready))
+
     def one(mode, lps=1, ctas=0):
-        """Enqueue one prefill under schedule `mode`; the main stream ends after it."""
+        """Enqueue one prefill under schedule `mode` ("fp8_" + mode: fp8 chunks); the main
+        stream ends after it."""
+        fp8 = mode.startswith("fp8_")
+        mode = mode[4:] if fp8 else mode
+        retrieve_all, store_all, retrieve_layers, store_layers = copies(fp8)
         start = ev()
         start.record(main)
         side.wait_event(start)
@@ -1076,14 +1099,14 @@ def run_layerwise(args):
             for _ in range(L):
                 torch.matmul(a, b, out=c)
         elif mode == "serial":
-            kvs.kvs_retrieve(g, buf.plane_ptrs, w.num_blocks, buf.requests, side, 0)
+            retrieve_all()
             done = ev()
             done.record(side)
             main.wait_event(done)
             for _ in range(L):
                 torch.matmul(a, b, out=c)
         elif mode == "retrieve":
-            kvs.kvs_retrieve(g, buf.plane_ptrs, w.num_blocks, buf.requests, side, 0)
+            retrieve_all()
             done = ev()
             done.record(side)
             main.wait_event(done)
@@ -1093,7 +1116,7 @@ def run_layerwise(args):
             computed = ev()
             computed.record(main)
             side.wait_event(computed)
-            kvs.kvs_store(g, buf.plane_ptrs, w.num_blocks, buf.store_requests, side, 0)
+            store_all()
             done = ev()
             done.record(side)
             main.wait_event(done)
@@ -1103,8 +1126,7 @@ def run_layerwise(args):
                 torch.matmul(a, b, out=c)
                 ready.append(ev())
                 ready[-1].record(main)
-            kvs.kvs_store_layers(g, buf.plane_ptrs, w.num_blocks, buf.store_requests, lps, None, side,
-                                 kvs.KVS_F_MAX_CTAS(ctas), ready_events=ready[lps - 1::lps] if lps > 1 else ready)
+            store_layers(lps, kvs.KVS_F_MAX_CTAS(ctas), ready[lps - 1::lps] if lps > 1 else ready)
             done = ev()
             done.record(side)
             main.wait_event(done)
@@ -1112,7 +1134,7 @@ def run_layerwise(args):
             groups = -(-L // lps)
             evs = [ev() for _ in range(groups)]
             fl = (kvs.KVS_F_LAYER_SIGNAL if mode == "signal" else 0) | kvs.KVS_F_MAX_CTAS(ctas)
-            kvs.kvs_retrieve_layers(g, buf.plane_ptrs, w.num_blocks, buf.requests, lps, evs, side, fl)
+            retrieve_layers(lps, evs, fl)
             for l in range(L):
                 if l % lps == 0:
                     main.wait_event(evs[l // lps])
@@ -1127,7 +1149,12 @@ def run_layerwise(args):
                  ("layerwise_signal_lps1_ctas16", "signal", 1, 16),
                  # store-back of the computed suffix: after the whole prefill, or layer by layer
                  ("store_serial", "store_serial", 1, 0), ("store_layerwise_lps1", "store_layer", 1, 0),
-                 ("store_layerwise_lps1_ctas4", "store_layer", 1, 4)]
+                 ("store_layerwise_lps1_ctas4", "store_layer", 1, 4),
+                 # the same with fp8 chunks: half the bytes over the link
+                 ("fp8_serial", "fp8_serial", 1, 0), ("fp8_layerwise_lps1", "fp8_layer", 1, 0),
+                 ("fp8_store_serial", "fp8_store_serial", 1, 0), ("fp8_store_layerwise_lps1", "fp8_store_layer", 1, 0),
+                 ("fp8_store_layerwise_lps1_ctas4", "fp8_store_layer", 1, 4),
+                 ("fp8_store_layerwise_lps1_ctas32", "fp8_store_layer", 1, 32)]
     reps = max(3, min(args.steps, 10))
     sampler = ClockSampler(0)
     time.sleep(0.2)

@@ -269,7 +269,10 @@ int kvs_store_fp8(const kvs_geometry* geom, const kvs_paged_cache* cache,
 /* Layer-wise forms of the two fp8 calls, with the semantics of kvs_retrieve_layers
  * / kvs_store_layers (the model can start on layer group k once layer_events[k]
  * fires; group k of a store waits on ready_events[k]): one launch per layer
- * group and source class, on cuda_stream.  KVS_F_LAYER_SIGNAL is not accepted. */
+ * group and source class, on cuda_stream.  Layer by layer, host-chunk stores
+ * run on the host-link store cap (see kvs_bw_report.store_ctas; KVS_F_MAX_CTAS
+ * overrides it), so that each group's launch leaves most SMs to the compute
+ * producing the next layers.  KVS_F_LAYER_SIGNAL is not accepted. */
 int kvs_retrieve_fp8_layers(const kvs_geometry* geom, const kvs_paged_cache* cache,
                             const kvs_request* requests, int32_t num_requests,
                             int32_t layers_per_step, void* const* layer_events,

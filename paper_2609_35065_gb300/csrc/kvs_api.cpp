@@ -959,8 +959,12 @@ int fp8_call(const kvs_geometry* g, const kvs_paged_cache* cache, const kvs_requ
             if (f.job.num_pieces >= (1ull << 31)) return fail(KVS_ERR_INVALID_ARG, "call too large: split it");
             // Retrieval: a CTA keeps up to 32 KiB of codes in flight, half a link-kernel
             // CTA's bytes, so it takes twice the link kernel's grid.  Store-back: one CTA
-            // per (chunk, plane, head) over the whole GPU.
-            const int grid = cap ? cap : (retrieve ? 2 * st.hostlink_ctas : 0);
+            // per (chunk, plane, head) over the whole GPU for a whole call (193 GB/s, the
+            // D2H link); layer by layer it runs beside the compute that produces the KV,
+            // where a whole-GPU launch per group displaces that compute, so it takes the
+            // host-link store cap (exposed store time per 8B prefill: 7.7 ms uncapped,
+            // 2.1 ms at 32 CTAs).
+            const int grid = cap ? cap : retrieve ? 2 * st.hostlink_ctas : layers_per_step > 0 ? st.store_ctas : 0;
             rc = run(f, grid);
             if (rc) return rc;
         }
