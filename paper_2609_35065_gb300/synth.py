@@ -107,7 +107,7 @@ def llama8b(requests: int = 16, prompt: int = 4096, hit: float = 0.5, num_blocks
     tables = _consecutive_tables(_perm(num_blocks, 0), [nb_each] * requests)
     matched = int(prompt * hit) // g.chunk_tokens * g.chunk_tokens
     reqs = [Request(prompt, matched, t, "host") for t in tables]
-    name = "llama8b" if (requests, num_blocks) == (16, 20000) else f"llama8b_r{requests}_nb{num_blocks}"
+    name = "llama8b" if (requests, num_blocks) == (16, 20000) else f"llama8b_{requests}req_nb{num_blocks}"
     return Workload(name, g, num_blocks, reqs)
 
 
@@ -150,7 +150,7 @@ def qwen14b(requests: int = 8, prompt: int = 16384, hit: float = 0.75,
         raise ValueError("not enough blocks")
     reqs = [Request(prompt, matched, t, "host", store_tokens=prompt - matched,
                     shared_prefix_tokens=shared_blocks * B) for t in tables]
-    name = "qwen14b" if (requests, num_blocks) == (8, 8192) else f"qwen14b_r{requests}_nb{num_blocks}"
+    name = "qwen14b" if (requests, num_blocks) == (8, 8192) else f"qwen14b_{requests}req_nb{num_blocks}"
     return Workload(name, g, num_blocks, reqs, notes={"shared_blocks": shared_blocks})
 
 

@@ -253,3 +253,22 @@ def test_fp8_layerwise_argument_checks():
         with pytest.raises(kvs.KvsError) as ei:
             fn(w.geom, buf.plane_ptrs, w.num_blocks, buf.requests, 1, None, None, kvs.KVS_F_LAYER_SIGNAL)
         assert ei.value.code == kvs.KVS_ERR_UNSUPPORTED
+
+
+@pytest.mark.parametrize("D,B", [(48, 3), (80, 16), (176, 1)])
+def test_fp8_head_dims_that_are_not_powers_of_two(D, B):
+    """head_dim 48 / 80 / 176 (3, 5 and 11 vectors of 16 codes per head): the retrieval's
+    per-vector head arithmetic and the two-pass store (D/8 does not divide the CTA), with
+    B = 3 and B = 1 paged blocks and a ragged last chunk, both residencies."""
+    C = 48 if B == 3 else 64
+    w = synth.custom(2, 3, D, B, C, 400, [200, 150], [150, 100], seed=D, residency=["host", "device"],
+                     store_tokens=[0, 0])
+    for r in w.requests:
+        r.store_tokens, r.store_first = r.matched_tokens, r.first_token
+    buf = buffers.allocate_fp8(w, store=True)
+    _retrieve(buf)
+    torch.cuda.synchronize()
+    gc.check_retrieve_fp8(buf)
+    _store(buf)
+    torch.cuda.synchronize()
+    gc.check_store_fp8(buf)
