@@ -29,7 +29,8 @@ if ROOT not in sys.path:
 METRIC = "prefix-KV retrieval GB/s and tokens/s on 1 GB300; % of HBM / host-link roofline"
 MEASURED_PEAKS = os.path.join(ROOT, "MEASURED_PEAKS.json")
 TRAFFIC_FILE = os.path.join(ROOT, "profiles", "traffic.json")
-KERNEL_SRC = os.path.join(ROOT, "paper_2609_35065_gb300", "csrc", "kvs_kernels.cu")
+# the copy kernels and the async-copy helpers they inline
+KERNEL_SRCS = [os.path.join(ROOT, "paper_2609_35065_gb300", "csrc", f) for f in ("kvs_kernels.cu", "kvs_async.cuh")]
 HBM_FALLBACK_GBS = 6800.0
 
 
@@ -113,8 +114,10 @@ def kernel_hash(src: str | None = None) -> str:
     with the code, not with its commentary."""
     import re
     if src is None:
-        with open(KERNEL_SRC) as f:
-            src = f.read()
+        src = ""
+        for path in KERNEL_SRCS:
+            with open(path) as f:
+                src += f.read() + "\n"
     src = re.sub(r"/\*.*?\*/", " ", src, flags=re.S)
     src = re.sub(r"//[^\n]*", " ", src)
     return hashlib.sha256(" ".join(src.split()).encode()).hexdigest()[:16]

@@ -19,7 +19,7 @@ OUT_DIR = os.path.join(PKG, "_build")
 LIB = os.path.join(OUT_DIR, "libkvs.so")
 SOURCES = [os.path.join(CSRC, f) for f in ("kvs_kernels.cu", "kvs_api.cpp", "kvs_noalloc.cu", "kvs_fp8.cu",
                                            "kvs_tier.cpp")]
-DEPS = SOURCES + [os.path.join(CSRC, "kvs_internal.h"), os.path.join(INCLUDE, "kvs.h")]
+DEPS = SOURCES + [os.path.join(CSRC, "kvs_internal.h"), os.path.join(CSRC, "kvs_async.cuh"), os.path.join(INCLUDE, "kvs.h")]
 ARCH = "-gencode=arch=compute_103a,code=sm_103a"
 
 

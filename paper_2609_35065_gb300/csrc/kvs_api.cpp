@@ -939,9 +939,13 @@ int fp8_call(const kvs_geometry* g, const kvs_paged_cache* cache, const kvs_requ
         f.block_magic = g->block_size >= 2 ? (uint32_t)((1ull << 32) / (uint64_t)g->block_size + 1) : 0;
         return f;
     };
-    auto run = [&](const Fp8Job& f, int grid) -> int {
+    // store-back segments: one per (chunk, plane, head)
+    auto fp8_segments = [](const Fp8Job& f) {
+        return (uint64_t)f.job.num_entries * f.job.num_planes * f.heads;
+    };
+    auto run = [&](const Fp8Job& f, int grid, bool device_chunks) -> int {
         cudaError_t e = retrieve ? launch_fp8_retrieve(f, grid, s)
-                                 : launch_fp8_store(f, grid, s, (uint32_t)g->chunk_tokens);
+                                 : launch_fp8_store(f, grid, s, (uint32_t)g->chunk_tokens, device_chunks);
         if (e != cudaSuccess) return fail(KVS_ERR_CUDA, "fp8 kernel launch failed: %s", cudaGetErrorString(e));
         ++g_launches;
         return KVS_OK;
@@ -956,7 +960,8 @@ int fp8_call(const kvs_geometry* g, const kvs_paged_cache* cache, const kvs_requ
             KVS_CUDA(cudaStreamWaitEvent(s, (cudaEvent_t)ready_events[k], 0));
         if (pl.num_host) {
             const Fp8Job f = fjob(pl.num_device, pl.num_host, p0, np);
-            if (f.job.num_pieces >= (1ull << 31)) return fail(KVS_ERR_INVALID_ARG, "call too large: split it");
+            if (f.job.num_pieces >= (1ull << 31) || fp8_segments(f) >= (1ull << 31))
+                return fail(KVS_ERR_INVALID_ARG, "call too large: split it");
             // Retrieval: a CTA keeps up to 32 KiB of codes in flight, half a link-kernel
             // CTA's bytes, so it takes twice the link kernel's grid.  Store-back: one CTA
             // per (chunk, plane, head) over the whole GPU for a whole call (193 GB/s, the
@@ -965,14 +970,16 @@ int fp8_call(const kvs_geometry* g, const kvs_paged_cache* cache, const kvs_requ
             // host-link store cap (exposed store time per 8B prefill: 7.7 ms uncapped,
             // 2.1 ms at 32 CTAs).
             const int grid = cap ? cap : retrieve ? 2 * st.hostlink_ctas : layers_per_step > 0 ? st.store_ctas : 0;
-            rc = run(f, grid);
+            rc = run(f, grid, false);
             if (rc) return rc;
         }
         if (pl.num_device) {
             const Fp8Job f = fjob(0, pl.num_device, p0, np);
-            if (f.job.num_pieces >= (1ull << 31)) return fail(KVS_ERR_INVALID_ARG, "call too large: split it");
-            // HBM chunks: uncapped retrievals run one CTA per piece
-            rc = run(f, cap ? cap : (retrieve ? kFp8PerPiece : 0));
+            if (f.job.num_pieces >= (1ull << 31) || fp8_segments(f) >= (1ull << 31))
+                return fail(KVS_ERR_INVALID_ARG, "call too large: split it");
+            // HBM chunks: uncapped retrievals run one CTA per piece, store-backs stage
+            // heads through shared memory
+            rc = run(f, cap ? cap : (retrieve ? kFp8PerPiece : 0), true);
             if (rc) return rc;
         }
         if (layers_per_step > 0 && layer_events && layer_events[k])

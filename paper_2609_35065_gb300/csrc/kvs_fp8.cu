@@ -30,10 +30,12 @@
 // scales of a piece's plane are loaded once per piece by H threads (one 4-byte
 // load each, beside the codes) and shared through shared memory, instead of
 // one scale load per vector; HBM chunks run one CTA per piece instead.
-// Store-back runs one 256-thread CTA per (chunk, plane, head): the head's BF16
-// elements are loaded into registers at once, reduced to the amax and
-// quantised from registers (heads too large for that take a two-pass kernel,
-// one CTA per (chunk, plane)).
+// Store-back to pinned host runs one 256-thread CTA per (chunk, plane, head):
+// the head's BF16 elements are loaded into registers at once, reduced to the
+// amax and quantised from registers (heads too large for that take a two-pass
+// kernel, one CTA per (chunk, plane)).  Into HBM chunks a persistent CTA per SM
+// stages heads in shared memory with per-thread async copies, two heads ahead
+// of the one it quantises.
 #include <cuda_bf16.h>
 #include <cuda_fp16.h>
 #include <cuda_fp8.h>
@@ -42,6 +44,7 @@
 #include <cstdint>
 
 #include "kvs.h"
+#include "kvs_async.cuh"
 #include "kvs_internal.h"
 
 namespace kvs {
@@ -211,17 +214,26 @@ __global__ void __launch_bounds__(kRtThreads, 8) kvs_fp8_retrieve_piece_kernel(c
 // Store-back (quantise)
 // ---------------------------------------------------------------------------
 
-// Per-halfword running maximum of |x| over the finite BF16 values of a
-// 32-bit word pair (|x| of a finite BF16 orders like its bits with the sign
-// cleared; infinities and NaN, exponent all ones, count as 0).
+// Per-halfword running maximum of |x| over the finite BF16 values of a word
+// pair.  |x| of a finite BF16 orders like its bits with the sign cleared
+// (0x0000..0x7F7F); adding 0x80 to each half moves the finite ones to
+// 0x0080..0x7FFF and infinities / NaN (0x7F80..0x7FFF) to 0x8000..0x807F,
+// negative as signed 16-bit lanes, so a signed lane maximum that starts from 0
+// never takes them (no carry crosses halves: each half stays below 0x10000).
+// The running value is offset by 0x80; amax_bits removes the offset.
 __device__ __forceinline__ uint32_t amax2(uint32_t m2, uint32_t w) {
-    const uint32_t a = w & 0x7FFF7FFFu;
-    return __vmaxu2(m2, a & ~__vcmpgeu2(a, 0x7F807F80u));
+    uint32_t r;
+    asm("max.s16x2 %0, %1, %2;" : "=r"(r) : "r"(m2), "r"((w & 0x7FFF7FFFu) + 0x00800080u));   // sm_90+
+    return r;
+}
+
+// Bits of the largest finite |x| (0 when there is none) from a running amax2 value.
+__device__ __forceinline__ uint32_t amax_bits(uint32_t m2) {
+    return max(max(m2 & 0xFFFFu, m2 >> 16), 0x80u) - 0x80u;
 }
 
 __device__ __forceinline__ uint32_t amax_bits8(const uint4& v) {
-    uint32_t m2 = amax2(amax2(amax2(amax2(0u, v.x), v.y), v.z), v.w);
-    return max(m2 & 0xFFFFu, m2 >> 16);
+    return amax_bits(amax2(amax2(amax2(amax2(0u, v.x), v.y), v.z), v.w));
 }
 
 __device__ __forceinline__ float bf16_lo(uint32_t w) { return __uint_as_float(w << 16); }
@@ -294,7 +306,7 @@ __device__ __forceinline__ void store_head_segment(const Fp8Job& f, uint32_t e, 
     for (int u = 0; u < kHeadVec; ++u)
         m2 = amax2(amax2(amax2(amax2(m2, v[u].x), v[u].y), v[u].z), v[u].w);
     if (bad) atomicCAS(j.err, 0, KVS_ERR_BOUNDS);
-    const uint32_t m = __reduce_max_sync(0xFFFFFFFFu, max(m2 & 0xFFFFu, m2 >> 16));
+    const uint32_t m = __reduce_max_sync(0xFFFFFFFFu, amax_bits(m2));
     if ((threadIdx.x & 31) == 0) warp_max[threadIdx.x >> 5] = m;
     __syncthreads();
     if (threadIdx.x == 0) {
@@ -332,6 +344,243 @@ __global__ void __launch_bounds__(kStThreads) kvs_fp8_store_head_kernel(const Fp
         else
             store_head_segment<false>(f, e, p, h, warp_max, &sm_inv);
     }
+}
+
+// ---------------------------------------------------------------------------
+// Staged store-back for HBM destinations: per-thread async copies
+// ---------------------------------------------------------------------------
+// A persistent 512-thread CTA per SM walks segments (as above, one (chunk,
+// plane, head) each).  Thread t owns the 16-byte column w = t % (D/8) of
+// tokens t / (D/8) + u * step, u < kSgVec (step = kSgThreads / (D/8)); its
+// loads go through shared memory: it copies its vectors of segment k with
+// cp.async into its own slots of stage k % kSgStages, kSgStages - 1 segments
+// ahead of the one it quantises, so two heads' loads (128 KiB) are in flight
+// per SM while its registers hold only the current head's 8 vectors.  A thread
+// reads back only the slots it filled itself, so the stages need no CTA
+// barrier (cp.async.wait_group orders them); the amax reduction takes two.
+// Slot u of thread t in a stage is at (u * kSgThreads + t) * 16.  The plane
+// rows of a full segment depend only on its chunk, so a thread keeps them in
+// registers while consecutive segments share the chunk.
+constexpr int kSgThreads = 512;
+constexpr int kSgVec = 8;
+constexpr int kSgStages = 3;
+constexpr uint32_t kSgStageBytes = kSgVec * kSgThreads * 16;        // 64 KiB
+constexpr uint32_t kSgSmemBytes = kSgStages * kSgStageBytes;
+static_assert(kSgStageBytes == kHeadMaxElems * 2, "a stage holds the largest single-pass head");
+
+// A CTA's segments are one contiguous range, walked with a cursor over
+// (entry, plane, head): consecutive segments share the chunk (and its plane
+// rows) and mostly the plane, and need no division to decode.
+struct SgCur {
+    uint32_t e, p, h;
+};
+
+__device__ __forceinline__ SgCur sg_at(const Fp8Job& f, uint32_t seg) {
+    const Job& j = f.job;
+    const uint32_t eh = seg / f.heads, h = seg - eh * f.heads;
+    const uint32_t e = eh / j.num_planes;
+    return {e, j.plane_begin + (eh - e * j.num_planes), h};
+}
+
+__device__ __forceinline__ void sg_step(const Fp8Job& f, SgCur& c) {
+    if (++c.h == f.heads) {
+        c.h = 0;
+        if (++c.p == f.job.plane_begin + f.job.num_planes) {
+            c.p = f.job.plane_begin;
+            ++c.e;
+        }
+    }
+}
+
+__device__ __forceinline__ void cp_async16(uint32_t dst_smem, uint64_t src) {
+    asm volatile("cp.async.cg.shared.global [%0], [%1], 16;" :: "r"(dst_smem), "l"(src) : "memory");
+}
+
+__device__ __forceinline__ void cp_async_commit() {
+    asm volatile("cp.async.commit_group;" ::: "memory");
+}
+
+template <int N>
+__device__ __forceinline__ void cp_async_wait() {
+    asm volatile("cp.async.wait_group %0;" :: "n"(N) : "memory");
+}
+
+__device__ __forceinline__ uint4 lds16(uint32_t a) {
+    uint4 r;
+    asm volatile("ld.shared.v4.u32 {%0,%1,%2,%3}, [%4];" : "=r"(r.x), "=r"(r.y), "=r"(r.z), "=r"(r.w) : "r"(a));
+    return r;
+}
+
+__device__ __forceinline__ void sts16_zero(uint32_t a) {
+    asm volatile("st.shared.v4.u32 [%0], {%1,%1,%1,%1};" :: "r"(a), "r"(0u) : "memory");
+}
+
+// Two BF16 (one word) times `inv` -> two E4M3 codes, with one packed binary32
+// multiply (sm_100+; each lane rounded to nearest like __fmul_rn).
+__device__ __forceinline__ uint32_t e4m3x2_of_pk(uint32_t w, uint64_t inv2) {
+    const uint64_t x2 = ((uint64_t)(w & 0xFFFF0000u) << 32) | (uint64_t)(w << 16);
+    uint64_t q2;
+    asm("mul.rn.f32x2 %0, %1, %2;" : "=l"(q2) : "l"(x2), "l"(inv2));
+    return (uint32_t)__nv_cvt_float2_to_fp8x2(
+        make_float2(__uint_as_float((uint32_t)q2), __uint_as_float((uint32_t)(q2 >> 32))), __NV_SATFINITE, __NV_E4M3);
+}
+
+__device__ __forceinline__ uint2 quant8_pk(const uint4& a, uint64_t inv2) {
+    return make_uint2(e4m3x2_of_pk(a.x, inv2) | (e4m3x2_of_pk(a.y, inv2) << 16),
+                      e4m3x2_of_pk(a.z, inv2) | (e4m3x2_of_pk(a.w, inv2) << 16));
+}
+
+// Plane row (blk * B + token % B) of token i of a chunk, or kNoRow for a bad block.
+constexpr uint32_t kNoRow = 0xFFFFFFFFu;
+
+__device__ __forceinline__ uint32_t sg_row(const Fp8Job& f, const int32_t* blocks, uint32_t i) {
+    const Job& j = f.job;
+    const uint32_t B = j.block_size;
+    const uint32_t bi = B == 1 ? i : __umulhi(i, f.block_magic);
+    const int32_t blk = __ldg(blocks + bi);
+    return (blk < 0 || blk >= j.num_blocks) ? kNoRow : (uint32_t)blk * B + (i - bi * B);
+}
+
+// This thread's loads of segment c (n tokens) into its slots of the stage at
+// `stage`; a bad block's vectors are zeros (and the call reports the error).
+// `rows` / `rows_e`: the cached rows of full segments and the chunk they belong to.
+template <bool FULL>
+__device__ __forceinline__ void sg_issue(const Fp8Job& f, const SgCur& c, uint32_t n, uint32_t stage,
+                                         uint32_t (&rows)[kSgVec], uint32_t& rows_e) {
+    const Job& j = f.job;
+    const uint32_t D = f.head_dim, vpt = D / 8, step = kSgThreads / vpt;
+    const uint32_t w = threadIdx.x % vpt, i0 = threadIdx.x / vpt;
+    const uint64_t row2 = (uint64_t)f.heads * D * 2;
+    const int32_t* blocks = j.blocks + (size_t)(j.entry_base + c.e) * j.blocks_per_chunk;
+    const uint64_t src0 = j.planes[c.p] + (uint64_t)c.h * D * 2 + (uint64_t)w * 16;
+    const uint32_t slot0 = stage + threadIdx.x * 16;
+    if (FULL && rows_e != c.e) {
+#pragma unroll
+        for (int u = 0; u < kSgVec; ++u) rows[u] = sg_row(f, blocks, i0 + u * step);
+        rows_e = c.e;
+    }
+    bool bad = false;
+#pragma unroll
+    for (int u = 0; u < kSgVec; ++u) {
+        const uint32_t i = i0 + u * step;
+        if (FULL || i < n) {
+            const uint32_t row = FULL ? rows[u] : sg_row(f, blocks, i);
+            const uint32_t slot = slot0 + u * kSgThreads * 16;
+            if (row == kNoRow) {
+                bad = true;
+                sts16_zero(slot);
+            } else {
+                cp_async16(slot, src0 + (uint64_t)row * row2);
+            }
+        }
+    }
+    if (bad) atomicCAS(j.err, 0, KVS_ERR_BOUNDS);
+}
+
+// Running max of |x| over BF16 pairs in one instruction (sm_86+): the result's
+// magnitude is the larger magnitude, its sign the XOR of the signs (cleared at
+// the end); a NaN input is ignored.  Infinities are not: a head whose maximum
+// comes out infinite takes the exact finite amax (amax2) instead.
+__device__ __forceinline__ uint32_t absmax2(uint32_t m2, uint32_t w) {
+    uint32_t r;
+    asm("max.xorsign.abs.bf16x2 %0, %1, %2;" : "=r"(r) : "r"(m2), "r"(w));
+    return r;
+}
+
+constexpr uint32_t kBf16Inf = 0x7F80u;
+
+// Quantises segment c (n tokens) from this thread's slots of `stage` (its loads
+// complete).  One barrier: every warp reads all warps' maxima (from the half of
+// warp_max this segment's parity selects) and computes the reciprocal itself;
+// a head holding an infinity takes one more barrier for its finite amax.
+template <bool FULL>
+__device__ __forceinline__ void sg_quantise(const Fp8Job& f, const SgCur& c, uint32_t n, uint32_t stage,
+                                            uint32_t* warp_max, uint32_t* warp_max_fin) {
+    const Job& j = f.job;
+    const uint32_t H = f.heads, D = f.head_dim, vpt = D / 8, step = kSgThreads / vpt;
+    const uint32_t t = threadIdx.x, w = t % vpt, i0 = t / vpt;
+    const uint32_t slot0 = stage + t * 16;
+    uint4 v[kSgVec];
+#pragma unroll
+    for (int u = 0; u < kSgVec; ++u) {
+        v[u] = make_uint4(0, 0, 0, 0);
+        if (FULL || i0 + u * step < n) v[u] = lds16(slot0 + u * kSgThreads * 16);
+    }
+    uint32_t x2 = 0;
+#pragma unroll
+    for (int u = 0; u < kSgVec; ++u)
+        x2 = absmax2(absmax2(absmax2(absmax2(x2, v[u].x), v[u].y), v[u].z), v[u].w);
+    x2 &= 0x7FFF7FFFu;                                      // never NaN: at most kBf16Inf per half
+    uint32_t m = __reduce_max_sync(0xFFFFFFFFu, max(x2 & 0xFFFFu, x2 >> 16));
+    if ((t & 31) == 0) warp_max[t >> 5] = m;
+    __syncthreads();
+    uint32_t a = __reduce_max_sync(0xFFFFFFFFu, warp_max[(t & 31) % (kSgThreads / 32)]);
+    if (a == kBf16Inf) {                                    // uniform across the CTA
+        uint32_t m2 = 0;
+#pragma unroll
+        for (int u = 0; u < kSgVec; ++u)
+            m2 = amax2(amax2(amax2(amax2(m2, v[u].x), v[u].y), v[u].z), v[u].w);
+        m = __reduce_max_sync(0xFFFFFFFFu, amax_bits(m2));
+        if ((t & 31) == 0) warp_max_fin[t >> 5] = m;
+        __syncthreads();
+        a = __reduce_max_sync(0xFFFFFFFFu, warp_max_fin[(t & 31) % (kSgThreads / 32)]);
+    }
+    const float af = __uint_as_float(a << 16);
+    const float inv = af > 0.0f ? __fdiv_rn(448.0f, af) : 1.0f;
+    const uint64_t chunk = j.entries[c.e].chunk;
+    if (t == 0) *reinterpret_cast<float*>(chunk + ((uint64_t)c.p * H + c.h) * 4) = af > 0.0f ? __fdiv_rn(af, 448.0f) : 1.0f;
+    const uint64_t inv2 = ((uint64_t)__float_as_uint(inv) << 32) | __float_as_uint(inv);
+    const uint64_t hd = (uint64_t)H * D;
+    const uint64_t codes = chunk + f.scale_bytes + (uint64_t)c.p * n * hd + (uint64_t)c.h * D + (uint64_t)w * 8 +
+                           (uint64_t)i0 * hd;
+#pragma unroll
+    for (int u = 0; u < kSgVec; ++u)
+        if (FULL || i0 + u * step < n) st_cs8(codes + (uint64_t)(u * step) * hd, quant8_pk(v[u], inv2));
+}
+
+// CTA b takes segments [b * N / G, (b + 1) * N / G).  warp_max has two halves,
+// alternating by segment: a warp writes a half again only two segments later,
+// after the next segment's barrier, which every warp reaches only once it has
+// read this segment's half.  warp_max_fin (heads holding an infinity) is
+// written after a segment's first barrier and read before its next one.
+static_assert(kSgThreads / 32 <= 32, "one lane per warp maximum");
+__global__ void __launch_bounds__(kSgThreads, 1) kvs_fp8_store_staged_kernel(const Fp8Job f, uint32_t num_segments) {
+    extern __shared__ __align__(128) uint8_t sg_stage[];
+    __shared__ uint32_t warp_max[2][kSgThreads / 32];
+    __shared__ uint32_t warp_max_fin[kSgThreads / 32];
+    const uint32_t base = smem_u32(sg_stage);
+    const uint32_t full_n = kSgVec * (kSgThreads / (f.head_dim / 8));
+    const uint32_t lo = (uint32_t)((uint64_t)blockIdx.x * num_segments / gridDim.x);
+    const uint32_t hi = (uint32_t)((uint64_t)(blockIdx.x + 1) * num_segments / gridDim.x);
+    if (lo >= hi) return;                                   // uniform across the CTA
+    const Entry* entries = f.job.entries;
+    uint32_t rows[kSgVec];
+    uint32_t rows_e = 0xFFFFFFFFu;
+    SgCur ic = sg_at(f, lo), qc = ic;                       // issue / quantise cursors
+    uint32_t issued = 0;
+    // one commit group per segment slot, empty past the end, so wait_group counts segments
+    auto issue = [&]() {
+        if (lo + issued < hi) {
+            const uint32_t n = (uint32_t)entries[ic.e].n_tok;
+            const uint32_t stage = base + (issued % kSgStages) * kSgStageBytes;
+            if (n == full_n) sg_issue<true>(f, ic, n, stage, rows, rows_e);
+            else sg_issue<false>(f, ic, n, stage, rows, rows_e);
+            sg_step(f, ic);
+            ++issued;
+        }
+        cp_async_commit();
+    };
+    for (int s = 0; s + 1 < kSgStages; ++s) issue();
+    for (uint32_t k = 0; lo + k < hi; ++k) {
+        issue();
+        cp_async_wait<kSgStages - 1>();
+        const uint32_t n = (uint32_t)entries[qc.e].n_tok;
+        const uint32_t stage = base + (k % kSgStages) * kSgStageBytes;
+        if (n == full_n) sg_quantise<true>(f, qc, n, stage, warp_max[k & 1], warp_max_fin);
+        else sg_quantise<false>(f, qc, n, stage, warp_max[k & 1], warp_max_fin);
+        sg_step(f, qc);
+    }
+    cp_async_wait<0>();
 }
 
 constexpr int kStUnroll = 4;                         // vectors per thread in flight per step
@@ -433,6 +682,8 @@ __global__ void __launch_bounds__(kStThreads) kvs_fp8_store_kernel(const Fp8Job 
 }
 
 int g_sms = 0;
+constexpr int kMaxDev = 64;
+bool g_sg_attr[kMaxDev];                 // dynamic shared memory limit of the staged store raised
 
 int sm_count() {
     if (g_sms == 0) {
@@ -462,12 +713,28 @@ cudaError_t launch_fp8_retrieve(const Fp8Job& fj, int grid, cudaStream_t s) {
     return cudaGetLastError();
 }
 
-cudaError_t launch_fp8_store(const Fp8Job& fj, int grid, cudaStream_t s, uint32_t chunk_tokens) {
+cudaError_t launch_fp8_store(const Fp8Job& fj, int grid, cudaStream_t s, uint32_t chunk_tokens, bool staged) {
     const uint32_t vpt = fj.head_dim / 8;
     if ((uint64_t)chunk_tokens * fj.head_dim <= kHeadMaxElems && kStThreads % vpt == 0 && chunk_tokens < 65536 &&
         fj.job.block_size < 65536) {
         const uint64_t segs = (uint64_t)fj.job.num_entries * fj.job.num_planes * fj.heads;
         if (segs == 0) return cudaSuccess;
+        // the staged kernel needs D/8 to divide its CTA and plane rows below 2^32 - 1
+        if (staged && kSgThreads % vpt == 0 && (uint64_t)fj.job.num_blocks * fj.job.block_size < 0xFFFFFFFFull) {
+            int dev = 0;
+            cudaGetDevice(&dev);
+            if (dev < 0 || dev >= kMaxDev) dev = 0;
+            if (!g_sg_attr[dev]) {
+                const cudaError_t e = cudaFuncSetAttribute(kvs_fp8_store_staged_kernel,
+                                                           cudaFuncAttributeMaxDynamicSharedMemorySize, kSgSmemBytes);
+                if (e != cudaSuccess) return e;
+                g_sg_attr[dev] = true;
+            }
+            if (grid <= 0 || grid > sm_count()) grid = sm_count();
+            if ((uint64_t)grid > segs) grid = (int)segs;
+            kvs_fp8_store_staged_kernel<<<grid, kSgThreads, kSgSmemBytes, s>>>(fj, (uint32_t)segs);
+            return cudaGetLastError();
+        }
         if (grid <= 0 || (uint64_t)grid > segs) grid = (int)std::min<uint64_t>(segs, 1u << 30);
         kvs_fp8_store_head_kernel<<<grid, kStThreads, 0, s>>>(fj, (uint32_t)segs);
         return cudaGetLastError();

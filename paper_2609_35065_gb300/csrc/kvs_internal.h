@@ -93,7 +93,9 @@ cudaError_t launch_fp8_retrieve(const Fp8Job& fj, int grid, cudaStream_t s);
 // Store-back: one CTA per (entry, plane, head) in a single pass when a head's
 // chunk_tokens x head_dim elements fit the CTA's registers, else one CTA per
 // (entry, plane) in two passes; a grid-stride loop over them with `grid` > 0.
-cudaError_t launch_fp8_store(const Fp8Job& fj, int grid, cudaStream_t s, uint32_t chunk_tokens);
+// `staged` (HBM destinations): the single pass runs as a persistent CTA per SM
+// (at most `grid` > 0) that stages heads in shared memory with bulk copies.
+cudaError_t launch_fp8_store(const Fp8Job& fj, int grid, cudaStream_t s, uint32_t chunk_tokens, bool staged);
 // Codes per retrieval piece (16 KiB).
 constexpr uint32_t kFp8PieceCodes = 16384;
 

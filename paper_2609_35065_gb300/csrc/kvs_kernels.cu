@@ -23,6 +23,7 @@
 #include <cstdint>
 
 #include "kvs.h"
+#include "kvs_async.cuh"
 #include "kvs_internal.h"
 
 namespace kvs {
@@ -428,70 +429,6 @@ __global__ void __launch_bounds__(kLdgThreads) kvs_flat_copy_kernel(uint64_t dst
 // TMA flavour: bulk async copies through a ring of shared-memory stages.
 // ---------------------------------------------------------------------------
 constexpr int kTmaStages = 6;
-constexpr uint64_t kWaitLimitNs = 2000000000ull;   // 2 s per wait: far above any piece
-
-__device__ __forceinline__ uint64_t global_ns() {
-    uint64_t t;
-    asm volatile("mov.u64 %0, %%globaltimer;" : "=l"(t));
-    return t;
-}
-
-__device__ __forceinline__ uint32_t smem_u32(const void* p) {
-    return (uint32_t)__cvta_generic_to_shared(p);
-}
-
-__device__ __forceinline__ void mbar_init(uint32_t bar, uint32_t count) {
-    asm volatile("mbarrier.init.shared::cta.b64 [%0], %1;" :: "r"(bar), "r"(count) : "memory");
-}
-
-__device__ __forceinline__ void mbar_expect_tx(uint32_t bar, uint32_t bytes) {
-    asm volatile("mbarrier.arrive.expect_tx.shared::cta.b64 _, [%0], %1;" :: "r"(bar), "r"(bytes) : "memory");
-}
-
-__device__ __forceinline__ bool mbar_try_wait(uint32_t bar, uint32_t parity) {
-    uint32_t ok;
-    asm volatile(
-        "{\n\t.reg .pred p;\n\t"
-        "mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2;\n\t"
-        "selp.u32 %0, 1, 0, p;\n\t}"
-        : "=r"(ok) : "r"(bar), "r"(parity) : "memory");
-    return ok != 0;
-}
-
-// Bounded wait: false once `limit_ns` has passed without the phase completing.
-__device__ __forceinline__ bool mbar_wait(uint32_t bar, uint32_t parity, uint64_t limit_ns) {
-    if (mbar_try_wait(bar, parity)) return true;
-    const uint64_t t0 = global_ns();
-    while (!mbar_try_wait(bar, parity)) {
-        if (global_ns() - t0 > limit_ns) return false;
-    }
-    return true;
-}
-
-__device__ __forceinline__ void bulk_load(uint32_t dst_smem, uint64_t src, uint32_t bytes, uint32_t bar) {
-    asm volatile(
-        "cp.async.bulk.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1], %2, [%3];"
-        :: "r"(dst_smem), "l"(src), "r"(bytes), "r"(bar) : "memory");
-}
-
-__device__ __forceinline__ void bulk_store(uint64_t dst, uint32_t src_smem, uint32_t bytes) {
-    asm volatile("cp.async.bulk.global.shared::cta.bulk_group [%0], [%1], %2;"
-                 :: "l"(dst), "r"(src_smem), "r"(bytes) : "memory");
-}
-
-__device__ __forceinline__ void bulk_commit() {
-    asm volatile("cp.async.bulk.commit_group;" ::: "memory");
-}
-
-template <int N>
-__device__ __forceinline__ void bulk_wait_read() {
-    asm volatile("cp.async.bulk.wait_group.read %0;" :: "n"(N) : "memory");
-}
-
-__device__ __forceinline__ void bulk_wait_all() {
-    asm volatile("cp.async.bulk.wait_group 0;" ::: "memory");
-}
-
 // One elected thread runs the whole pipeline: piece k of this CTA lives in
 // stage k % S; S-1 loads are kept in flight; before a stage is refilled the
 // bulk store that read it (one iteration earlier) must have finished reading.
@@ -505,7 +442,7 @@ __global__ void __launch_bounds__(32, 1) kvs_tma_kernel(const Decoder dc, uint32
     const bool to_plane = (j.mode == MODE_RETRIEVE);
 
     for (int s = 0; s < S; ++s) mbar_init(smem_u32(&bars[s]), 1);
-    asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+    mbar_init_fence();
 
     uint32_t cursor = blockIdx.x;
     auto next_piece = [&](Piece& out) -> bool {
@@ -568,7 +505,7 @@ __global__ void __launch_bounds__(32) kvs_tma_piece_kernel(const Decoder dc) {
     if (!decode_piece(dc, blockIdx.x, pc)) return;
     const uint32_t b = smem_u32(&bar);
     mbar_init(b, 1);
-    asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+    mbar_init_fence();
     mbar_expect_tx(b, pc.len);
     bulk_load(smem_u32(stage), MODE == MODE_RETRIEVE ? pc.chunk_addr : pc.plane_addr, pc.len, b);
     if (!mbar_wait(b, 0, kWaitLimitNs)) {
@@ -586,7 +523,7 @@ __global__ void kvs_stall_kernel(int32_t* err, uint64_t limit_ns) {
     __shared__ __align__(8) uint64_t bar;
     if (threadIdx.x != 0) return;
     mbar_init(smem_u32(&bar), 1);
-    asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+    mbar_init_fence();
     if (!mbar_wait(smem_u32(&bar), 0, limit_ns)) atomicCAS(err, 0, KVS_ERR_TIMEOUT);
 }
 

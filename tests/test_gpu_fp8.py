@@ -68,13 +68,15 @@ def _bf16(x):
     return np.array(x, dtype=np.float32).view(np.uint32) >> 16
 
 
-def test_fp8_special_values():
+@pytest.mark.parametrize("store_residency", ["host", "device"])
+def test_fp8_special_values(store_residency):
     """Retrieval: NaN codes, the largest codes, subnormal codes and signed zeros under
-    NaN, infinite, zero, subnormal and huge scales.  Store-back: planes holding NaN,
-    infinities, signed zeros, BF16 subnormals, values at exact midpoints between E4M3
-    codes (a head whose amax is 448 has scale 1), and magnitudes at and around 2^-10."""
+    NaN, infinite, zero, subnormal and huge scales.  Store-back (per-head register kernel
+    to pinned host, staged kernel to HBM): planes holding NaN, infinities, signed zeros,
+    BF16 subnormals, values at exact midpoints between E4M3 codes (a head whose amax is
+    448 has scale 1), and magnitudes at and around 2^-10."""
     w = synth.custom(2, 2, 32, 16, 32, 8, [64], [32], store_tokens=[32])
-    buf = buffers.allocate_fp8(w, store=True)
+    buf = buffers.allocate_fp8(w, store=True, store_residency=store_residency)
     ch = buf.chunks[0][0]
     # one scale per (plane, head): 4 planes x 2 heads
     scales = np.array([np.nan, np.inf, 0.0, 1e-40, 3e38, 1.0, -2.0, 0.5], dtype=np.float32)
@@ -106,15 +108,18 @@ def test_fp8_special_values():
     gc.check_store_fp8(buf)
 
 
-def test_fp8_llama8b_host_batch_retrieve_and_store():
+@pytest.mark.parametrize("store_residency", ["host", "device"])
+def test_fp8_llama8b_host_batch_retrieve_and_store(store_residency):
     """The 8B batch (16 requests x 2048 matched tokens, 128 chunks of 256 tokens: 2 GiB of
     codes + scale blocks in pinned host memory) dequantised into the 20,000-block cache,
-    then stored back into fresh pinned fp8 chunks; every plane and chunk against the oracle."""
+    then stored back into fresh fp8 chunks, pinned (the per-head register kernel) or in HBM
+    (the staged kernel, 65,536 heads over one CTA per SM); every plane and chunk against
+    the oracle."""
     w = synth.llama8b()
     for r in w.requests:
         r.store_tokens = r.matched_tokens
         r.store_first = 0
-    buf = buffers.allocate_fp8(w, store=True)
+    buf = buffers.allocate_fp8(w, store=True, store_residency=store_residency)
     assert buf.payload_bytes == 128 * (2048 + (16 << 20))
     s = torch.cuda.Stream()
     kvs.kvs_retrieve_fp8(w.geom, buf.plane_ptrs, w.num_blocks, buf.requests, s, 0)
@@ -269,6 +274,55 @@ def test_fp8_head_dims_that_are_not_powers_of_two(D, B):
     _retrieve(buf)
     torch.cuda.synchronize()
     gc.check_retrieve_fp8(buf)
+    _store(buf)
+    torch.cuda.synchronize()
+    gc.check_store_fp8(buf)
+
+
+@pytest.mark.parametrize("ctas", [1, 2, 7])
+def test_fp8_staged_store_with_few_ctas(ctas):
+    """HBM-destination store-back with 1, 2 and 7 CTAs: each CTA cycles its shared-memory
+    stages many times (stage reuse, barrier phases wrapping), over full chunks, a ragged
+    last chunk and a nonzero store start."""
+    w = synth.custom(3, 4, 128, 16, 256, 300, [1500, 1100], [0, 0], seed=ctas, store_tokens=[1200, 1000],
+                     firsts=[256, 0])
+    buf = buffers.allocate_fp8(w, store=True, store_residency="device")
+    gen = torch.Generator(device="cuda").manual_seed(ctas)
+    for p in range(buf.planes.shape[0]):
+        synth.fill_values(buf.planes[p], "normal", gen)
+    torch.cuda.synchronize()
+    _store(buf, kvs.KVS_F_VALIDATE | kvs.KVS_F_MAX_CTAS(ctas))
+    torch.cuda.synchronize()
+    gc.check_store_fp8(buf)
+
+
+@pytest.mark.parametrize("store_residency", ["host", "device"])
+def test_fp8_store_nan_without_infinity(store_residency):
+    """Heads holding NaNs of both signs (and no infinity) among normal values, heads of
+    zeros and BF16 subnormals only, and heads holding one infinity: the amax ignores the
+    NaNs and infinities, and every code and scale equals the oracle's."""
+    w = synth.custom(2, 8, 128, 16, 256, 64, [512], [0], seed=5, store_tokens=[512])
+    buf = buffers.allocate_fp8(w, store=True, store_residency=store_residency)
+    rng = np.random.default_rng(5)
+    for p in range(buf.planes.shape[0]):
+        vals = _bf16(rng.standard_normal(buf.planes[p].numel()).astype(np.float32)).astype(np.uint16)
+        vals = vals.reshape(-1, 8, 128)                       # [rows][head][d]
+        for h, kind in enumerate(["nan", "nan", "zero_sub", "inf", "nan_inf", "plain", "nan", "zero"]):
+            sel = vals[:, h, :].copy()
+            if kind.startswith("nan"):                        # ~2% NaNs of both signs
+                idx = rng.choice(sel.size, size=sel.size // 50, replace=False)
+                sel.reshape(-1)[idx] = rng.choice(np.array([0x7FC0, 0xFFC0, 0x7FC1, 0xFFFF, 0x7F81, 0xFF81],
+                                                           dtype=np.uint16), size=idx.size)
+            if kind.endswith("inf"):                          # ~0.05% infinities of both signs
+                idx = rng.choice(sel.size, size=sel.size // 2000, replace=False)
+                sel.reshape(-1)[idx] = rng.choice(np.array([0x7F80, 0xFF80], dtype=np.uint16), size=idx.size)
+            if kind == "zero_sub":
+                sel[:] = rng.choice(np.array([0x0000, 0x8000, 0x0001, 0x8003, 0x007F], dtype=np.uint16), size=sel.shape)
+            if kind == "zero":
+                sel[:] = 0
+            vals[:, h, :] = sel
+        buf.planes[p].copy_(torch.from_numpy(vals.reshape(-1).view(np.int16)))
+    torch.cuda.synchronize()
     _store(buf)
     torch.cuda.synchronize()
     gc.check_store_fp8(buf)
