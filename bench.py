@@ -42,7 +42,8 @@ def parse_args(argv=None):
     ap.add_argument("--impl", choices=["ours", "reference"], default="ours")
     ap.add_argument("--config", default="llama8b",
                     help="llama8b | sweep25 | sweep50 | sweep75 | qwen14b | llama70b[_25|_50|_100]")
-    ap.add_argument("--variant", choices=["auto", "hostlink", "hbmcopy"], default="auto")
+    ap.add_argument("--variant", choices=["auto", "hostlink", "hbmcopy", "few_sms"], default="auto",
+                    help="host-chunk variant; few_sms: KVS_F_FEW_SMS (staged host-link kernel, its own cap)")
     ap.add_argument("--kernel", choices=["auto", "ldg", "tma"], default="auto")
     ap.add_argument("--max-ctas", type=int, default=0)
     ap.add_argument("--probe-bytes", type=int, default=1 << 30)
@@ -363,6 +364,8 @@ def run_ours(args):
         flags |= kvs.KVS_F_FORCE_HOSTLINK
     elif args.variant == "hbmcopy":
         flags |= kvs.KVS_F_FORCE_HBMCOPY
+    elif args.variant == "few_sms":
+        flags |= kvs.KVS_F_FEW_SMS
     if args.kernel == "ldg":
         flags |= kvs.KVS_F_FORCE_LDG
     elif args.kernel == "tma":
@@ -370,7 +373,7 @@ def run_ours(args):
     if args.max_ctas:
         flags |= kvs.KVS_F_MAX_CTAS(args.max_ctas)
     choice = kvs.kvs_get_choice()
-    host_variant = {"hostlink": 1, "hbmcopy": 2}.get(args.variant, choice["chosen_retrieve_host"])
+    host_variant = {"hostlink": 1, "hbmcopy": 2, "few_sms": 1}.get(args.variant, choice["chosen_retrieve_host"])
 
     def step(requests, f=flags):
         kvs.kvs_retrieve(g, buf.plane_ptrs, w.num_blocks, requests, stream, f)
@@ -404,7 +407,8 @@ def run_ours(args):
     call_ms = statistics.mean(per_call_ms)
     value = whole_job_rate(payload, K, world, total_ms) / 1e9
     tokens_per_s = whole_job_rate(tokens, K, world, total_ms)
-    kernel_name = "kvs_link_kernel" if host_variant == 1 else "hbmcopy_pipeline"
+    kernel_name = ("kvs_link_staged_kernel" if args.variant == "few_sms" else "kvs_link_kernel") if host_variant == 1 \
+        else "hbmcopy_pipeline"
 
     # e2e: the public API from host arguments (request objects built anew each step),
     # each step's status word read back to the host.  Pipelined as a serving loop
@@ -787,7 +791,8 @@ def default_line_legs(args, buf, bw, stream, sampler, flags):
       20,000-block cache, with each source class alone;
     * ``overlap``: the 70B-shaped batch (pinned buffer of 25%, 4 passes, refilled
       between passes) retrieved on a high-priority side stream beside a bf16 8192^3
-      GEMM loop, at the default CTA cap.
+      GEMM loop: at the default CTA cap, with KVS_F_FEW_SMS (the staged kernel on its
+      measured cap), and as a plain copy-engine copy.
     """
     import torch
     from paper_2609_35065_gb300 import buffers, kvs, synth
@@ -897,10 +902,11 @@ def default_line_legs(args, buf, bw, stream, sampler, flags):
     w70 = synth.llama70b(buffer_frac=0.25)
     results, info = overlap_measure(w70, bw, side, [
         ("default", 0),
-        ("prefetch_l2_24ctas", kvs.KVS_F_PREFETCH_L2 | kvs.KVS_F_MAX_CTAS(24)),
+        ("few_sms", kvs.KVS_F_FEW_SMS),
         ("copy_engine_only", COPY_ENGINE_ONLY)], sampler)
-    legs["overlap"] = {"workload": describe(w70), **info, "hostlink_ctas": kvs.kvs_get_choice()["hostlink_ctas"],
-                       "side_stream": "high priority", **results}
+    choice = kvs.kvs_get_choice()
+    legs["overlap"] = {"workload": describe(w70), **info, "hostlink_ctas": choice["hostlink_ctas"],
+                       "few_sm_ctas": choice["few_sm_ctas"], "side_stream": "high priority", **results}
     return legs
 
 
@@ -1019,6 +1025,10 @@ def run_overlap(args):
                 ("hostlink_24ctas", kvs.KVS_F_FORCE_HOSTLINK | kvs.KVS_F_MAX_CTAS(24)),
                 ("hbmcopy", kvs.KVS_F_FORCE_HBMCOPY),
                 ("dma", kvs.KVS_F_FORCE_DMA),
+                ("few_sms", kvs.KVS_F_FEW_SMS),
+                ("few_sms_12ctas", kvs.KVS_F_FEW_SMS | kvs.KVS_F_MAX_CTAS(12)),
+                ("few_sms_16ctas", kvs.KVS_F_FEW_SMS | kvs.KVS_F_MAX_CTAS(16)),
+                ("few_sms_24ctas", kvs.KVS_F_FEW_SMS | kvs.KVS_F_MAX_CTAS(24)),
                 ("prefetch_l2_12ctas", kvs.KVS_F_PREFETCH_L2 | kvs.KVS_F_MAX_CTAS(12)),
                 ("prefetch_l2_24ctas", kvs.KVS_F_PREFETCH_L2 | kvs.KVS_F_MAX_CTAS(24)),
                 ("copy_engine_only", COPY_ENGINE_ONLY),
@@ -1030,6 +1040,7 @@ def run_overlap(args):
     line = {"metric": METRIC + " (overlap with a bf16 GEMM loop)", "unit": "GB/s",
             "config": {"workload": describe(w), **info},
             "side_stream_priority": args.side_priority, "hostlink_ctas_default": bw["hostlink_ctas"],
+            "few_sm_ctas_default": bw["few_sm_ctas"],
             "variants": results}
     print(json.dumps(line), flush=True)
     return 0

@@ -101,6 +101,18 @@ extern "C" {
                                           bulk L2 prefetches, so the bytes in flight wait
                                           in L2 rather than in registers and a small
                                           KVS_F_MAX_CTAS grid can hold the link rate      */
+#define KVS_F_FEW_SMS        (1u << 10) /* retrieval of host chunks on a GPU that runs other
+                                          kernels meanwhile (a model's compute): the
+                                          host-link variant with a kernel that holds
+                                          more bytes in flight per SM (one 32 KiB piece
+                                          in registers and three in shared memory per
+                                          256 threads, two CTAs per SM), on its own
+                                          measured cap (kvs_bw_report.few_sm_ctas), so
+                                          the link rate needs fewer SMs.  16-byte
+                                          aligned chunks, planes and rows (else the
+                                          plain host-link kernels run); not with
+                                          KVS_F_FORCE_HBMCOPY / _DMA, KVS_F_PREFETCH_L2
+                                          or KVS_F_LAYER_SIGNAL; store calls ignore it  */
 #define KVS_F_MAX_CTAS(n)    ((((uint32_t)(n)) & 0xFFFFu) << 16) /* cap on CTAs, 0 = auto */
 #define KVS_F_GET_MAX_CTAS(f) (((f) >> 16) & 0xFFFFu)
 
@@ -304,6 +316,12 @@ typedef struct kvs_bw_report {
     int64_t probe_bytes;           /* bytes moved per probe                                */
     double  retrieve_dma_gbs;      /* host-chunk retrieval probe, DMA variant              */
     double  store_dma_gbs;         /* host-chunk store probe, DMA variant                  */
+    int32_t few_sm_ctas;           /* CTA cap of KVS_F_FEW_SMS retrievals: 1.25 x the
+                                      smallest probed grid within 3% of the kernel's best
+                                      rate (before any kvs_query_bw: one per 8 SMs, at
+                                      least 8)                                             */
+    int32_t reserved;
+    double  few_sm_gbs;            /* best KVS_F_FEW_SMS retrieval probe rate              */
 } kvs_bw_report;
 
 /*
@@ -540,7 +558,7 @@ void* kvs_tier_slot(const kvs_tier* tier, int64_t slot);
 
 /* ABI version of this header: major * 10000 + minor * 100 + patch. */
 int kvs_version(void);
-#define KVS_VERSION 10800
+#define KVS_VERSION 10900
 
 #ifdef __cplusplus
 }

@@ -115,6 +115,7 @@ struct DevState {
     size_t       max_pitch = 0;              // largest pitch a 2D copy accepts
     int          hostlink_ctas = 0;          // CTA cap of host-link kernels, 0 = whole GPU
     int          store_ctas = 0;
+    int          few_sm_ctas = 0;            // CTA cap of KVS_F_FEW_SMS retrievals
     kvs_bw_report report{};
 };
 
@@ -166,9 +167,11 @@ int get_state(DevState** out) {
         // Until kvs_query_bw measures them, host-link kernels take a third of the
         // SMs' worth of CTAs: enough to saturate the link, not the whole GPU.
         st.hostlink_ctas = st.store_ctas = std::max(8, st.sms / 3);
+        st.few_sm_ctas = std::max(8, st.sms / 8);
         st.report.num_sms = st.sms;
         st.report.hostlink_ctas = st.hostlink_ctas;
         st.report.store_ctas = st.store_ctas;
+        st.report.few_sm_ctas = st.few_sm_ctas;
         st.report.chosen_retrieve_host = st.retrieve_host;
         st.report.chosen_store_host = st.store_host;
         st.report.chosen_kernel_device = st.kernel_device;
@@ -530,15 +533,19 @@ Job make_job(DevState& st, const kvs_geometry* g, const kvs_paged_cache* cache, 
     return j;
 }
 
-// Internal flavour: the double-buffered kernel used for host-resident chunks.
+// Internal flavours: the double-buffered kernel used for host-resident chunks,
+// with L2 prefetches, and with shared-memory stages (KVS_F_FEW_SMS).
 constexpr int kKernelLink = 100;
 constexpr int kKernelLinkPrefetch = 101;   // retrieval only
+constexpr int kKernelLinkStaged = 102;     // retrieval only
 
 int launch_kernel(const Job& j, int flavour, int vec, int grid, cudaStream_t s) {
     if (j.num_pieces == 0) return KVS_OK;
     cudaError_t e = (flavour == KVS_KERNEL_TMA) ? launch_tma(j, grid, s)
+                  : (flavour == kKernelLinkStaged && vec == 16) ? launch_link_staged(j, grid, s)
                   : (flavour == kKernelLinkPrefetch && vec == 16) ? launch_link_prefetch(j, grid, s)
-                  : ((flavour == kKernelLink || flavour == kKernelLinkPrefetch) && vec == 16) ? launch_link(j, grid, s)
+                  : ((flavour == kKernelLink || flavour == kKernelLinkPrefetch || flavour == kKernelLinkStaged) && vec == 16)
+                      ? launch_link(j, grid, s)
                   : launch_ldg(j, vec, grid, s);
     if (e != cudaSuccess) return fail(KVS_ERR_CUDA, "kernel launch failed: %s", cudaGetErrorString(e));
     ++g_launches;
@@ -702,6 +709,11 @@ int copy_call(const kvs_geometry* g, const kvs_paged_cache* cache, const kvs_req
     const bool f_ldg = flags & KVS_F_FORCE_LDG, f_tma = flags & KVS_F_FORCE_TMA;
     if ((int)f_host + (int)f_hbm + (int)f_dma > 1 || (f_ldg && f_tma))
         return fail(KVS_ERR_INVALID_ARG, "conflicting FORCE flags");
+    // KVS_F_FEW_SMS: host chunks over the host link, on the staged kernel (retrieval)
+    const bool f_few = retrieve && (flags & KVS_F_FEW_SMS);
+    if (f_few && (f_hbm || f_dma || (flags & (KVS_F_PREFETCH_L2 | KVS_F_LAYER_SIGNAL))))
+        return fail(KVS_ERR_INVALID_ARG, "KVS_F_FEW_SMS takes the host-link variant, without "
+                    "KVS_F_PREFETCH_L2 or KVS_F_LAYER_SIGNAL");
     if ((flags & KVS_F_LAYER_LAUNCHES) && (flags & KVS_F_LAYER_SIGNAL))
         return fail(KVS_ERR_INVALID_ARG, "KVS_F_LAYER_LAUNCHES and KVS_F_LAYER_SIGNAL together");
     if (ready_events && (flags & KVS_F_LAYER_SIGNAL))
@@ -740,8 +752,8 @@ int copy_call(const kvs_geometry* g, const kvs_paged_cache* cache, const kvs_req
         if (f_tma) return fail(KVS_ERR_UNSUPPORTED, "TMA needs 16-byte aligned chunks, planes and rows");
         flavour = KVS_KERNEL_LDG;
     }
-    int host_variant = f_host ? KVS_VARIANT_HOSTLINK : f_hbm ? KVS_VARIANT_HBMCOPY : f_dma ? KVS_VARIANT_DMA
-                                                            : (retrieve ? st.retrieve_host : st.store_host);
+    int host_variant = (f_host || f_few) ? KVS_VARIANT_HOSTLINK : f_hbm ? KVS_VARIANT_HBMCOPY
+                     : f_dma ? KVS_VARIANT_DMA : (retrieve ? st.retrieve_host : st.store_host);
     if (layers_per_step > 0) host_variant = KVS_VARIANT_HOSTLINK;
     uint64_t pitch = 0;
     if (host_variant == KVS_VARIANT_DMA && pl.num_host) {
@@ -753,7 +765,7 @@ int copy_call(const kvs_geometry* g, const kvs_paged_cache* cache, const kvs_req
         }
     }
     const Mode mode = retrieve ? MODE_RETRIEVE : MODE_STORE;
-    const int host_grid = grid ? grid : (retrieve ? st.hostlink_ctas : st.store_ctas);
+    const int host_grid = grid ? grid : f_few ? st.few_sm_ctas : (retrieve ? st.hostlink_ctas : st.store_ctas);
 
     Uploaded u;
     rc = upload(st, pl, s, u);
@@ -837,7 +849,8 @@ int copy_call(const kvs_geometry* g, const kvs_paged_cache* cache, const kvs_req
                 rc = host_variant == KVS_VARIANT_DMA ? run_dma(g, pl, pitch, retrieve, s, host_addr)
                                                      : run_hbmcopy(st, g, cache, pl, u, mode, flavour, grid, s, host_addr);
             } else {
-                const int lf = (retrieve && (flags & KVS_F_PREFETCH_L2)) ? kKernelLinkPrefetch : kKernelLink;
+                const int lf = f_few ? kKernelLinkStaged
+                             : (retrieve && (flags & KVS_F_PREFETCH_L2)) ? kKernelLinkPrefetch : kKernelLink;
                 rc = launch_kernel(make_job(st, g, cache, pl, u, pl.num_device, pl.num_host, mode, p0, np),
                                    lf, vec, host_grid, s);
             }
@@ -1126,11 +1139,29 @@ int query_bw(DevState& st, kvs_bw_report* out, cudaStream_t s, int64_t probe_byt
             if (dir == 0) rep.hostlink_ctas = pick; else rep.store_ctas = pick;
         }
     }
+    // KVS_F_FEW_SMS cap: 1.25 x the smallest grid within 3% of the staged
+    // kernel's best rate on an idle GPU.  Beside a bf16 GEMM loop that keeps the
+    // link at 96-98% on 8-10 SMs, where the plain kernel needs 16 or more.
+    {
+        const int cand[] = {8, 12, 16, 20, 24, 32};
+        double gb[6] = {}, best = 0;
+        for (int k = 0; k < 6; ++k) {
+            rc = probe_call(&rh, true, KVS_F_FEW_SMS | KVS_F_MAX_CTAS(cand[k]), &gb[k]);
+            if (rc) { cleanup(); return rc; }
+            best = std::max(best, gb[k]);
+        }
+        int pick = cand[5];
+        for (int k = 0; k < 6; ++k)
+            if (gb[k] >= 0.97 * best) { pick = cand[k]; break; }
+        rep.few_sm_ctas = (pick * 5 / 4 + 1) & ~1;
+        rep.few_sm_gbs = best;
+    }
 #undef PROBE
     KVS_CUDA(cudaStreamSynchronize(s));
     cleanup();
     st.hostlink_ctas = rep.hostlink_ctas;
     st.store_ctas = rep.store_ctas;
+    st.few_sm_ctas = rep.few_sm_ctas;
     // The probe's buffer is small.  On GB300 the copy engine's rate from pinned
     // host memory is erratic on buffers of tens of GiB (13-210 GB/s on 40 GiB,
     // by box and allocation), where SM loads keep the link's rate, so the
@@ -1382,6 +1413,7 @@ int kvs_get_choice(kvs_bw_report* out) {
     out->num_sms = st->sms;
     out->hostlink_ctas = st->hostlink_ctas;
     out->store_ctas = st->store_ctas;
+    out->few_sm_ctas = st->few_sm_ctas;
     return KVS_OK;
 }
 

@@ -55,6 +55,10 @@ cudaError_t launch_ldg(const Job& job, int vec_bytes, int grid, cudaStream_t s);
 cudaError_t launch_tma(const Job& job, int grid, cudaStream_t s);
 // Double-buffered 16-byte flavour for host-resident chunks (retrieve or store).
 cudaError_t launch_link(const Job& job, int grid, cudaStream_t s);
+// Retrieval of host chunks holding more bytes in flight per SM (one piece in
+// registers and three in shared memory per 256 threads, two CTAs per SM), for
+// GPUs that run other kernels meanwhile (KVS_F_FEW_SMS).
+cudaError_t launch_link_staged(const Job& job, int grid, cudaStream_t s);
 // The same for retrieval, with each CTA's upcoming pieces prefetched into L2.
 cudaError_t launch_link_prefetch(const Job& job, int grid, cudaStream_t s);
 // Contiguous copy of `bytes` (multiple of 16, 16-byte aligned) for bandwidth probes.

@@ -281,6 +281,98 @@ __global__ void __launch_bounds__(kLdgThreads) kvs_link_kernel(const Decoder dc,
     }
 }
 
+// Few-SM flavour of the host-link retrieval (KVS_F_FEW_SMS).  Beside a kernel
+// whose CTAs fill whole SMs (a GEMM), every SM that holds a copy CTA is lost to
+// it, so what matters is the bytes in flight per SM.  Each thread keeps one
+// piece in registers, as the link kernel does, and three more in shared
+// memory, copied there with cp.async into slots that only it reads back (no
+// CTA barrier; cp.async.wait_group orders them): 128 KiB per CTA and two CTAs
+// per SM, 256 KiB per SM against the link kernel's 192.  Piece i of a CTA
+// lives in slot i % 4 -- slot 0 the registers, slots 1-3 shared memory -- and
+// its successor i + 4 is issued into the slot as soon as piece i is stored.
+// Pieces come in grid-stride order, so once a slot finds none left, neither
+// does any slot after it.
+constexpr int kStagedSmemPieces = 3;
+constexpr int kStagedSlots = 1 + kStagedSmemPieces;
+constexpr uint32_t kStagedSmemBytes = kStagedSmemPieces * kPieceBytes;
+
+__device__ __forceinline__ void cp_async16(uint32_t dst_smem, uint64_t src) {
+    asm volatile("cp.async.cg.shared.global [%0], [%1], 16;" :: "r"(dst_smem), "l"(src) : "memory");
+}
+
+__device__ __forceinline__ void cp_async_commit() {
+    asm volatile("cp.async.commit_group;" ::: "memory");
+}
+
+template <int N>
+__device__ __forceinline__ void cp_async_wait() {
+    asm volatile("cp.async.wait_group %0;" :: "n"(N) : "memory");
+}
+
+// This thread's vectors of a piece into its slots of shared-memory stage `stage`.
+__device__ __forceinline__ void stage_piece16(uint64_t src, uint32_t len, uint32_t stage) {
+    const uint32_t n = len / 16;
+#pragma unroll
+    for (int u = 0; u < kLdgUnroll; ++u) {
+        const uint32_t k = threadIdx.x + u * kLdgThreads;
+        if (k < n) cp_async16(stage + k * 16, src + (uint64_t)k * 16);
+    }
+}
+
+// ... and from its slots to `dst` (the thread's own cp.async copies are complete).
+__device__ __forceinline__ void unstage_piece16(uint64_t dst, uint32_t len, uint32_t stage) {
+    const uint32_t n = len / 16;
+    uint4 v[kLdgUnroll];
+#pragma unroll
+    for (int u = 0; u < kLdgUnroll; ++u) {
+        const uint32_t k = threadIdx.x + u * kLdgThreads;
+        if (k < n)
+            asm volatile("ld.shared.v4.u32 {%0,%1,%2,%3}, [%4];"
+                         : "=r"(v[u].x), "=r"(v[u].y), "=r"(v[u].z), "=r"(v[u].w) : "r"(stage + k * 16));
+    }
+    store_piece16(dst, len, v);
+}
+
+__global__ void __launch_bounds__(kLdgThreads, 2) kvs_link_staged_kernel(const Decoder dc, uint32_t num_pieces) {
+    extern __shared__ __align__(128) uint8_t link_stage[];
+    const uint32_t base = smem_u32(link_stage);
+    uint4 r[kLdgUnroll];
+    Piece pc[kStagedSlots];
+    bool has[kStagedSlots];
+    uint32_t q = blockIdx.x;
+    // fill slot s with the CTA's next piece; a shared-memory slot always commits
+    // one group (empty past the end), so wait_group counts pieces
+    auto fill = [&](int s) {
+        has[s] = next_piece_ldg(dc, num_pieces, q, pc[s]);
+        if (s == 0) {
+            if (has[s]) load_piece16(pc[s].chunk_addr, pc[s].len, r);
+        } else {
+            if (has[s]) stage_piece16(pc[s].chunk_addr, pc[s].len, base + (s - 1) * kPieceBytes);
+            cp_async_commit();
+        }
+    };
+#pragma unroll
+    for (int s = 0; s < kStagedSlots; ++s) fill(s);
+    bool more = true;
+    while (more) {
+#pragma unroll
+        for (int s = 0; s < kStagedSlots; ++s) {
+            if (more && !has[s]) more = false;
+            if (more) {
+                if (s == 0) {
+                    store_piece16(pc[s].plane_addr, pc[s].len, r);
+                } else {
+                    // the kStagedSmemPieces - 1 younger shared-memory pieces may still be in flight
+                    cp_async_wait<kStagedSmemPieces - 1>();
+                    unstage_piece16(pc[s].plane_addr, pc[s].len, base + (s - 1) * kPieceBytes);
+                }
+                fill(s);
+            }
+        }
+    }
+    cp_async_wait<0>();
+}
+
 // L2-prefetch flavour of the host-link retrieval.  Over the host link a piece's
 // loads take ~15 us beside a busy GPU, so the plain flavour needs ~3 MiB of
 // loads in flight, held in registers: 16 or more SMs' worth of CTAs.  Here the
@@ -607,6 +699,25 @@ cudaError_t launch_link_prefetch(const Job& job, int grid, cudaStream_t s) {
     // about 4 MiB of prefetches in flight over the whole grid
     const uint32_t ahead = (uint32_t)std::min(64, std::max(2, (int)((4u << 20) / kPieceBytes) / grid));
     kvs_link_pf_kernel<<<grid, kLdgThreads, 0, s>>>(make_decoder(job), (uint32_t)job.num_pieces, ahead);
+    return cudaGetLastError();
+}
+
+int link_staged_ctas_per_sm() {
+    static int n = 0;
+    if (n == 0) {
+        cudaFuncSetAttribute(kvs_link_staged_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)kStagedSmemBytes);
+        cudaFuncSetAttribute(kvs_link_staged_kernel, cudaFuncAttributePreferredSharedMemoryCarveout, 100);
+        cudaOccupancyMaxActiveBlocksPerMultiprocessor(&n, kvs_link_staged_kernel, kLdgThreads, kStagedSmemBytes);
+        if (n <= 0) n = 1;
+    }
+    return n;
+}
+
+cudaError_t launch_link_staged(const Job& job, int grid, cudaStream_t s) {
+    if (job.num_pieces == 0) return cudaSuccess;
+    if (job.mode != MODE_RETRIEVE) return cudaErrorInvalidValue;
+    grid = clamp_grid(grid, link_staged_ctas_per_sm(), job.num_pieces);
+    kvs_link_staged_kernel<<<grid, kLdgThreads, kStagedSmemBytes, s>>>(make_decoder(job), (uint32_t)job.num_pieces);
     return cudaGetLastError();
 }
 

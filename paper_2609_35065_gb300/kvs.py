@@ -46,6 +46,7 @@ KVS_F_LAYER_LAUNCHES = 1 << 6
 KVS_F_LAYER_SIGNAL = 1 << 7
 KVS_F_FORCE_DMA = 1 << 8
 KVS_F_PREFETCH_L2 = 1 << 9
+KVS_F_FEW_SMS = 1 << 10
 KVS_DIR_RETRIEVE = 0
 KVS_DIR_STORE = 1
 
@@ -116,7 +117,8 @@ class kvs_bw_report(ctypes.Structure):
                 ("chosen_kernel_device", ctypes.c_int32), ("num_sms", ctypes.c_int32),
                 ("hostlink_ctas", ctypes.c_int32), ("store_ctas", ctypes.c_int32),
                 ("probe_bytes", ctypes.c_int64), ("retrieve_dma_gbs", ctypes.c_double),
-                ("store_dma_gbs", ctypes.c_double)]
+                ("store_dma_gbs", ctypes.c_double), ("few_sm_ctas", ctypes.c_int32), ("reserved", ctypes.c_int32),
+                ("few_sm_gbs", ctypes.c_double)]
 
     def as_dict(self) -> dict:
         out = {}

@@ -25,7 +25,7 @@ def test_library_exports_every_declared_function():
     for n in names:
         assert hasattr(lib, n), n
     assert set(names) == set(kvs.EXPORTED)
-    assert kvs.kvs_version() == 10800
+    assert kvs.kvs_version() == 10900
 
 
 def test_struct_layouts_match_header():
@@ -33,7 +33,7 @@ def test_struct_layouts_match_header():
     assert ctypes.sizeof(kvs.kvs_chunk) == 16
     assert ctypes.sizeof(kvs.kvs_request) == 40
     assert ctypes.sizeof(kvs.kvs_paged_cache) == 16
-    assert ctypes.sizeof(kvs.kvs_bw_report) == 5 * 8 + 6 * 8 + 6 * 4 + 8 + 2 * 8
+    assert ctypes.sizeof(kvs.kvs_bw_report) == 5 * 8 + 6 * 8 + 6 * 4 + 8 + 2 * 8 + 2 * 4 + 8
     assert ctypes.sizeof(kvs.kvs_tune_report) == 3 * 8 + 8 + 2 * 4 + 2 * 8 + 8 + 2 * 4
 
 
@@ -123,6 +123,25 @@ def test_malformed_calls_are_rejected(fn, case, code):
     got, msg = _code(fn=fn, **case)
     assert got == code, msg
     assert kvs.kvs_last_error() == msg.split(": ", 1)[1]
+
+
+@pytest.mark.parametrize("extra", [kvs.KVS_F_FORCE_HBMCOPY, kvs.KVS_F_FORCE_DMA, kvs.KVS_F_PREFETCH_L2],
+                         ids=["hbmcopy", "dma", "prefetch_l2"])
+def test_few_sms_retrieval_refuses_other_variants(extra):
+    """KVS_F_FEW_SMS selects the host-link variant on its own kernel: combined with a
+    copy-engine variant or the L2-prefetch kernel a retrieval is refused before any device
+    work; a store ignores the flag (its argument checks still run first)."""
+    got, msg = _code(fn=kvs.kvs_retrieve, flags=kvs.KVS_F_FEW_SMS | extra)
+    assert got == kvs.KVS_ERR_INVALID_ARG, msg
+    assert "KVS_F_FEW_SMS" in msg
+    got, msg = _code(fn=kvs.kvs_store, reqs=[_req(table=(0, 1, 8, 3))], flags=kvs.KVS_F_FEW_SMS | extra)
+    assert got == kvs.KVS_ERR_BOUNDS, msg
+
+
+def test_few_sms_layerwise_refuses_the_signalling_launch():
+    with pytest.raises(kvs.KvsError) as ei:
+        kvs.kvs_retrieve_layers(G, _planes(), 8, [_req()], 1, None, None, kvs.KVS_F_FEW_SMS | kvs.KVS_F_LAYER_SIGNAL)
+    assert ei.value.code == kvs.KVS_ERR_INVALID_ARG
 
 
 def test_null_base_pointer_is_rejected():

@@ -215,3 +215,64 @@ def test_prefetch_l2_random_small_geometries(seed):
     torch.cuda.synchronize()
     gc.check_retrieve(buf)
     gc.check_store(buf)
+
+
+@pytest.mark.parametrize("cap", [0, 1, 5, 20], ids=["default_grid", "1_cta", "5_ctas", "20_ctas"])
+def test_few_sms_retrieval(cap):
+    """KVS_F_FEW_SMS (one piece per thread in registers, three in shared memory): the 8B
+    shape (2 requests, 512 MiB) and a ragged multi-piece shape, every element checked;
+    one CTA cycles its four slots thousands of times."""
+    flags = kvs.KVS_F_FEW_SMS | kvs.KVS_F_VALIDATE | kvs.KVS_F_MAX_CTAS(cap)
+    for w in (synth.llama8b(requests=2, num_blocks=1024),
+              synth.custom(2, 8, 256, 16, 256, 300, [1024, 700, 512], [1024, 700, 512], seed=6, dist="normal")):
+        buf = buffers.allocate(w)
+        kvs.kvs_retrieve(w.geom, buf.plane_ptrs, w.num_blocks, buf.requests, None, flags)
+        torch.cuda.synchronize()
+        gc.check_retrieve(buf)
+        gc.free(buf)
+
+
+@pytest.mark.parametrize("seed", range(8))
+def test_few_sms_random_small_geometries(seed):
+    """Random geometries with mixed residency: 16-byte host rows take the staged kernel,
+    the rest the vector kernel, device chunks their own kernels; stores ignore the flag."""
+    w = gc.random_workload(seed)
+    buf = buffers.allocate(w, store=True, store_residency="host")
+    flags = kvs.KVS_F_FEW_SMS | kvs.KVS_F_VALIDATE | kvs.KVS_F_MAX_CTAS(seed % 4)
+    kvs.kvs_retrieve(w.geom, buf.plane_ptrs, w.num_blocks, buf.requests, None, flags)
+    kvs.kvs_store(w.geom, buf.plane_ptrs, w.num_blocks, buf.store_requests, None, flags)
+    torch.cuda.synchronize()
+    gc.check_retrieve(buf)
+    gc.check_store(buf)
+
+
+def test_few_sms_layerwise_groups_and_probe():
+    """Layer-wise KVS_F_FEW_SMS retrieval (one staged launch per layer group) fires each
+    group's event after exactly the oracle's planes of that group; kvs_query_bw then
+    reports the staged kernel's cap and rate, and calls without a cap use it."""
+    w = synth.custom(6, 8, 128, 16, 256, 200, [1024, 768], [1024, 768], seed=9)
+    g = w.geom
+    buf = buffers.allocate(w)
+    events = [torch.cuda.Event() for _ in range(3)]
+    copier, consumer = torch.cuda.Stream(), torch.cuda.Stream()
+    kvs.kvs_retrieve_layers(g, buf.plane_ptrs, w.num_blocks, buf.requests, 2, events, copier, kvs.KVS_F_FEW_SMS)
+    snaps = []
+    for k, ev in enumerate(events):
+        consumer.wait_event(ev)
+        with torch.cuda.stream(consumer):
+            snaps.append(buf.planes[4 * k:4 * k + 4].clone())
+    torch.cuda.synchronize()
+    assert kvs.kvs_check_errors(None) == kvs.KVS_OK
+    chunks_np = gc.host_chunks(buf)
+    for k, snap in enumerate(snaps):
+        for i in range(4):
+            want = gc.expected_plane(buf, 4 * k + i, chunks_np)
+            assert np.array_equal(snap[i].cpu().numpy().view(want.dtype), want), (k, i)
+    rep = kvs.kvs_query_bw(None, 256 << 20)
+    assert 10 <= rep["few_sm_ctas"] <= 40 and rep["few_sm_ctas"] % 2 == 0, rep["few_sm_ctas"]
+    assert rep["few_sm_gbs"] > 0
+    assert kvs.kvs_get_choice()["few_sm_ctas"] == rep["few_sm_ctas"]
+    _sentinel(buf)
+    kvs.kvs_retrieve(g, buf.plane_ptrs, w.num_blocks, buf.requests, None, kvs.KVS_F_FEW_SMS | kvs.KVS_F_VALIDATE)
+    gc.check_retrieve(buf)
+    kvs.kvs_shutdown()
