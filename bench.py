@@ -1147,7 +1147,8 @@ def run_layerwise(args):
         else:
             groups = -(-L // lps)
             evs = [ev() for _ in range(groups)]
-            fl = (kvs.KVS_F_LAYER_SIGNAL if mode == "signal" else 0) | kvs.KVS_F_MAX_CTAS(ctas)
+            fl = ((kvs.KVS_F_LAYER_SIGNAL if mode == "signal" else kvs.KVS_F_FEW_SMS if mode == "layer_few" else 0)
+                  | kvs.KVS_F_MAX_CTAS(ctas))
             retrieve_layers(lps, evs, fl)
             for l in range(L):
                 if l % lps == 0:
@@ -1155,12 +1156,14 @@ def run_layerwise(args):
                 torch.matmul(a, b, out=c)
 
     # "layer": the default (one launch per layer group); "signal": one resident
-    # launch that signals each group (KVS_F_LAYER_SIGNAL)
+    # launch that signals each group (KVS_F_LAYER_SIGNAL); "layer_few": one launch
+    # per group on the staged few-SM kernel (KVS_F_FEW_SMS)
     schedules = [("compute_only", "compute", 1, 0), ("serial", "serial", 1, 0),
                  ("layerwise_lps1", "layer", 1, 0), ("layerwise_lps4", "layer", 4, 0),
                  ("layerwise_lps8", "layer", 8, 0), ("layerwise_lps1_ctas4", "layer", 1, 4),
                  ("layerwise_signal_lps1", "signal", 1, 0), ("layerwise_signal_lps1_ctas4", "signal", 1, 4),
                  ("layerwise_signal_lps1_ctas16", "signal", 1, 16),
+                 ("layerwise_few_sms_lps1", "layer_few", 1, 0), ("layerwise_few_sms_lps1_ctas8", "layer_few", 1, 8),
                  # store-back of the computed suffix: after the whole prefill, or layer by layer
                  ("store_serial", "store_serial", 1, 0), ("store_layerwise_lps1", "store_layer", 1, 0),
                  ("store_layerwise_lps1_ctas4", "store_layer", 1, 4),
