@@ -626,6 +626,11 @@ def run_ours(args):
 COPY_ENGINE_ONLY = -1          # overlap variant: plain copy-engine copy of the pinned buffer, no scatter
 
 
+def FP8(flags: int = 0):
+    """Overlap variant: the same tokens retrieved from fp8 chunks (kvs_retrieve_fp8)."""
+    return ("fp8", flags)
+
+
 def overlap_measure(w, bw, side, variants, sampler=None):
     """Retrieval of workload ``w`` on the ``side`` stream while the current stream runs a
     bf16 8192 x 8192 GEMM loop, for each (name, flags) of ``variants``, alone and beside the
@@ -653,6 +658,30 @@ def overlap_measure(w, bw, side, variants, sampler=None):
     del src
     refill_src = pinned.clone() if passes > 1 else None      # stands in for the next pass's KV
     C = g.chunk_tokens
+    fp8_chunk_bytes = 2 * g.layers * C * g.row_elems + (2 * g.layers * g.kv_heads * 4 + 255) // 256 * 256
+
+    fp8 = {}
+
+    def fp8_requests(k):
+        """The pass's tokens as fp8 chunks in one pinned pool (built on first use)."""
+        from paper_2609_35065_gb300 import buffers
+        if "pool" not in fp8:
+            cb = (buffers.fp8_chunk_bytes(g, C) + 255) // 256 * 256
+            fp8["cb"] = cb
+            fp8["pool"] = torch.empty((tokens_pass // C) * cb, dtype=torch.uint8, pin_memory=True)
+            gen = torch.Generator(device="cuda").manual_seed(w.seed)
+            for j in range(tokens_pass // C):
+                buffers.fill_fp8_chunk(fp8["pool"][j * cb:(j + 1) * cb], g, gen)
+            fp8["refill"] = fp8["pool"].clone() if passes > 1 else None
+        cb, pool = fp8["cb"], fp8["pool"]
+        reqs, at = [], 0
+        for r in w.requests[k * per_pass:(k + 1) * per_pass]:
+            cs = []
+            for j in range(r.matched_tokens // C):
+                cs.append(kvs.ChunkArg(pool[at:at + buffers.fp8_chunk_bytes(g, C)], C))
+                at += cb
+            reqs.append(kvs.RequestArg(r.block_table, cs))
+        return reqs
 
     def pass_requests(k):
         reqs, at = [], 0
@@ -720,6 +749,9 @@ def overlap_measure(w, bw, side, variants, sampler=None):
         (a layer-wise call without events), which hands SMs back between layers.  The
         flags value COPY_ENGINE_ONLY instead copies the pass's pinned buffer into one HBM
         buffer with a plain cudaMemcpyAsync: the copy engine's rate with no scatter."""
+        if isinstance(flags, tuple):
+            kvs.kvs_retrieve_fp8(g, ptrs, w.num_blocks, reqs, side, flags[1])
+            return
         if flags == COPY_ENGINE_ONLY:
             if "dst" not in scratch:
                 scratch["dst"] = torch.empty_like(pinned, device="cuda")
@@ -734,10 +766,14 @@ def overlap_measure(w, bw, side, variants, sampler=None):
     def retrieval(flags, with_gemm):
         total_ms, gemm_during, gemm_alone = 0.0, [], []
         wall = [time.time(), None]
+        is_fp8 = isinstance(flags, tuple)
         for k in range(passes):
-            if k:
-                pinned.copy_(refill_src)                 # refill between passes (untimed)
-            reqs = pass_requests(k)
+            reqs = fp8_requests(k) if is_fp8 else pass_requests(k)
+            if k:                                        # refill between passes (untimed)
+                if is_fp8:
+                    fp8["pool"].copy_(fp8["refill"])
+                else:
+                    pinned.copy_(refill_src)
             copy(reqs, flags)                            # warm
             torch.cuda.synchronize()
             if not with_gemm:
@@ -757,8 +793,10 @@ def overlap_measure(w, bw, side, variants, sampler=None):
             a0, aev, _ = gemm_window(iters)
             gemm_alone.append(rate_within(a0, aev, r_ms))
         wall[1] = time.time()
-        gbs = passes * tokens_pass * per_tok * 2 / (total_ms / 1e3) / 1e9
-        out = {"retrieval_gbs": round(gbs, 2), "frac_of_host_link": round(gbs / host_peak, 4)}
+        moved = tokens_pass // C * fp8_chunk_bytes if is_fp8 else tokens_pass * per_tok * 2
+        gbs = passes * moved / (total_ms / 1e3) / 1e9
+        out = {"retrieval_gbs": round(gbs, 2), "frac_of_host_link": round(gbs / host_peak, 4),
+               "tokens_per_s": round(passes * tokens_pass / (total_ms / 1e3), 1)}
         if with_gemm:
             during, alone = statistics.mean(gemm_during), statistics.mean(gemm_alone)
             out.update({"gemm_tflops_during": round(during, 1), "gemm_tflops_alone_same_window": round(alone, 1),
@@ -775,6 +813,7 @@ def overlap_measure(w, bw, side, variants, sampler=None):
             "gemm_tflops_short_burst": round(2 * 8192 ** 3 / (gemm_ms / 1e3) / 1e12, 1)}
     del planes, pinned, refill_src, a, b, c
     scratch.clear()
+    fp8.clear()
     torch.cuda.empty_cache()
     return results, info
 
@@ -792,7 +831,8 @@ def default_line_legs(args, buf, bw, stream, sampler, flags):
     * ``overlap``: the 70B-shaped batch (pinned buffer of 25%, 4 passes, refilled
       between passes) retrieved on a high-priority side stream beside a bf16 8192^3
       GEMM loop: at the default CTA cap, with KVS_F_FEW_SMS (the staged kernel on its
-      measured cap), and as a plain copy-engine copy.
+      measured cap), from fp8 chunks of the same tokens (``tokens_per_s`` compares them;
+      default grid and KVS_F_FEW_SMS), and as a plain copy-engine copy.
     """
     import torch
     from paper_2609_35065_gb300 import buffers, kvs, synth
@@ -903,6 +943,8 @@ def default_line_legs(args, buf, bw, stream, sampler, flags):
     results, info = overlap_measure(w70, bw, side, [
         ("default", 0),
         ("few_sms", kvs.KVS_F_FEW_SMS),
+        ("fp8", FP8()),
+        ("fp8_few_sms", FP8(kvs.KVS_F_FEW_SMS)),
         ("copy_engine_only", COPY_ENGINE_ONLY)], sampler)
     choice = kvs.kvs_get_choice()
     legs["overlap"] = {"workload": describe(w70), **info, "hostlink_ctas": choice["hostlink_ctas"],
@@ -931,6 +973,8 @@ def run_fp8(args):
     fb = buffers.allocate_fp8(w, store=True)
     fbytes = fb.payload_bytes
     flags = kvs.KVS_F_MAX_CTAS(args.max_ctas) if args.max_ctas else 0
+    if args.variant == "few_sms":
+        flags |= kvs.KVS_F_FEW_SMS
 
     def timed(fn, k):
         evs = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)) for _ in range(k)]
@@ -1029,6 +1073,11 @@ def run_overlap(args):
                 ("few_sms_12ctas", kvs.KVS_F_FEW_SMS | kvs.KVS_F_MAX_CTAS(12)),
                 ("few_sms_16ctas", kvs.KVS_F_FEW_SMS | kvs.KVS_F_MAX_CTAS(16)),
                 ("few_sms_24ctas", kvs.KVS_F_FEW_SMS | kvs.KVS_F_MAX_CTAS(24)),
+                ("fp8", FP8()), ("fp8_few_sms", FP8(kvs.KVS_F_FEW_SMS)),
+                ("fp8_few_sms_12ctas", FP8(kvs.KVS_F_FEW_SMS | kvs.KVS_F_MAX_CTAS(12))),
+                ("fp8_few_sms_8ctas", FP8(kvs.KVS_F_FEW_SMS | kvs.KVS_F_MAX_CTAS(8))),
+                ("fp8_48ctas", FP8(kvs.KVS_F_MAX_CTAS(48))),
+                ("fp8_24ctas", FP8(kvs.KVS_F_MAX_CTAS(24))), ("fp8_12ctas", FP8(kvs.KVS_F_MAX_CTAS(12))),
                 ("prefetch_l2_12ctas", kvs.KVS_F_PREFETCH_L2 | kvs.KVS_F_MAX_CTAS(12)),
                 ("prefetch_l2_24ctas", kvs.KVS_F_PREFETCH_L2 | kvs.KVS_F_MAX_CTAS(24)),
                 ("copy_engine_only", COPY_ENGINE_ONLY),

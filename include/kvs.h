@@ -101,16 +101,18 @@ extern "C" {
                                           bulk L2 prefetches, so the bytes in flight wait
                                           in L2 rather than in registers and a small
                                           KVS_F_MAX_CTAS grid can hold the link rate      */
-#define KVS_F_FEW_SMS        (1u << 10) /* retrieval of host chunks on a GPU that runs other
-                                          kernels meanwhile (a model's compute): the
-                                          host-link variant with a kernel that holds
-                                          more bytes in flight per SM (one 32 KiB piece
-                                          in registers and three in shared memory per
-                                          256 threads, two CTAs per SM), on its own
-                                          measured cap (kvs_bw_report.few_sm_ctas), so
-                                          the link rate needs fewer SMs.  16-byte
-                                          aligned chunks, planes and rows (else the
-                                          plain host-link kernels run); not with
+#define KVS_F_FEW_SMS        (1u << 10) /* retrieval of host chunks on a GPU that runs
+                                          other kernels meanwhile (a model's compute):
+                                          the host-link variant with a kernel that holds
+                                          more bytes in flight per SM (BF16: one 32 KiB
+                                          piece in registers and three in shared memory
+                                          per 256 threads; fp8: two 16 KiB pieces of
+                                          codes in registers and five in shared memory;
+                                          two CTAs per SM), on its own measured cap
+                                          (kvs_bw_report.few_sm_ctas), so the link rate
+                                          needs fewer SMs.  BF16: 16-byte aligned
+                                          chunks, planes and rows (else the plain
+                                          host-link kernels run); not with
                                           KVS_F_FORCE_HBMCOPY / _DMA, KVS_F_PREFETCH_L2
                                           or KVS_F_LAYER_SIGNAL; store calls ignore it  */
 #define KVS_F_MAX_CTAS(n)    ((((uint32_t)(n)) & 0xFFFFu) << 16) /* cap on CTAs, 0 = auto */
@@ -251,9 +253,11 @@ int kvs_store_layers(const kvs_geometry* geom, const kvs_paged_cache* cache,
  * a multiple of 16, H at most 128, chunks and planes 16-byte aligned
  * (KVS_ERR_UNSUPPORTED otherwise).  Arguments, layouts of the planes and
  * block tables, residencies, asynchrony and errors are as for kvs_retrieve /
- * kvs_store; the accepted flags are KVS_F_VALIDATE, KVS_F_MAX_CTAS (and
+ * kvs_store; the accepted flags are KVS_F_VALIDATE, KVS_F_MAX_CTAS,
+ * KVS_F_FEW_SMS (retrieval: host chunks on a kernel holding more codes in
+ * flight per SM, on kvs_bw_report.few_sm_ctas; stores ignore it) and
  * KVS_F_FORCE_HOSTLINK / KVS_F_FORCE_LDG, which name what always runs: host
- * chunks are read or written over the host link by SM loads and stores).
+ * chunks are read or written over the host link by SM loads and stores.
  *
  * kvs_retrieve_fp8: plane[2l+kv][slot(s_j+i)][h][d] =
  *     bf16(e4m3(code[l][kv][i][h][d]) * scale[l][kv][h]): the product is one
@@ -264,10 +268,10 @@ int kvs_store_layers(const kvs_geometry* geom, const kvs_paged_cache* cache,
  *     the chunks that hold them.
  * kvs_store_fp8: for every chunk, layer, K/V and head, amax = the largest |x|
  *     over the finite BF16 elements of the chunk's tokens (0 if none), scale =
- *     amax / 448 (binary32, nearest even; 1 when amax is 0), code = E4M3 of
- *     x / scale (binary32 division, nearest even), rounded to nearest even
- *     and saturated to +-448 (OFP8 saturation mode; infinities too); NaN
- *     elements give the code 0x7F.  The scales and codes of every destination
+ *     amax / 448 and inv = 448 / amax (binary32 divisions, nearest even; both
+ *     1 when amax is 0), code = E4M3 of x * inv (one binary32 multiply,
+ *     nearest even), rounded to nearest even and saturated to +-448 (OFP8
+ *     saturation mode; infinities too); NaN elements give the code 0x7F.  The scales and codes of every destination
  *     chunk are written; the cache is only read.
  */
 #define KVS_FP8_SCALE_BYTES(L, H) ((((int64_t)2 * (L) * (H) * 4) + 255) / 256 * 256)

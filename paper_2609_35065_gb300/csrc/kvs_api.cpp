@@ -891,10 +891,11 @@ int copy_call(const kvs_geometry* g, const kvs_paged_cache* cache, const kvs_req
 int fp8_call(const kvs_geometry* g, const kvs_paged_cache* cache, const kvs_request* reqs,
              int32_t nreq, void* stream, uint32_t flags, bool retrieve, int32_t layers_per_step = 0,
              void* const* layer_events = nullptr, void* const* ready_events = nullptr) {
-    const uint32_t allowed = KVS_F_VALIDATE | KVS_F_FORCE_HOSTLINK | KVS_F_FORCE_LDG | 0xFFFF0000u;
+    const uint32_t allowed = KVS_F_VALIDATE | KVS_F_FORCE_HOSTLINK | KVS_F_FORCE_LDG | KVS_F_FEW_SMS | 0xFFFF0000u;
     if (flags & ~allowed)
         return fail(KVS_ERR_UNSUPPORTED, "fp8 calls take only KVS_F_VALIDATE, KVS_F_FORCE_HOSTLINK, "
-                    "KVS_F_FORCE_LDG and KVS_F_MAX_CTAS");
+                    "KVS_F_FORCE_LDG, KVS_F_FEW_SMS and KVS_F_MAX_CTAS");
+    const bool few = retrieve && (flags & KVS_F_FEW_SMS);
     Plan pl;
     int rc = validate_call(g, cache, reqs, nreq, pl);
     if (rc) return rc;
@@ -950,6 +951,16 @@ int fp8_call(const kvs_geometry* g, const kvs_paged_cache* cache, const kvs_requ
         f.scale_bytes = (uint32_t)fp8_scale_bytes(g);
         // floor(2^32 / B) + 1 fits 32 bits for B >= 2; the kernel divides by B = 1 itself
         f.block_magic = g->block_size >= 2 ? (uint32_t)((1ull << 32) / (uint64_t)g->block_size + 1) : 0;
+        auto recip = [](uint32_t d, uint32_t& m, uint32_t& p) {
+            uint32_t l = 0;
+            while ((1ull << l) < d) ++l;
+            p = 31 + l;
+            m = (uint32_t)(((1ull << p) + d - 1) / d);
+        };
+        recip(f.job.pieces_per_run, f.ppr_m, f.ppr_p);
+        recip(f.job.num_planes * f.job.blocks_per_chunk, f.pe_m, f.pe_p);
+        recip(f.job.blocks_per_chunk, f.bpc_m, f.bpc_p);
+        f.rows_whole = (kFp8PieceCodes / 16) % (hd / 16) == 0;
         return f;
     };
     // store-back segments: one per (chunk, plane, head)
@@ -957,8 +968,9 @@ int fp8_call(const kvs_geometry* g, const kvs_paged_cache* cache, const kvs_requ
         return (uint64_t)f.job.num_entries * f.job.num_planes * f.heads;
     };
     auto run = [&](const Fp8Job& f, int grid, bool device_chunks) -> int {
-        cudaError_t e = retrieve ? launch_fp8_retrieve(f, grid, s)
-                                 : launch_fp8_store(f, grid, s, (uint32_t)g->chunk_tokens, device_chunks);
+        cudaError_t e = !retrieve ? launch_fp8_store(f, grid, s, (uint32_t)g->chunk_tokens, device_chunks)
+                      : (few && !device_chunks) ? launch_fp8_retrieve_staged(f, grid, s)
+                                                : launch_fp8_retrieve(f, grid, s);
         if (e != cudaSuccess) return fail(KVS_ERR_CUDA, "fp8 kernel launch failed: %s", cudaGetErrorString(e));
         ++g_launches;
         return KVS_OK;
@@ -982,7 +994,10 @@ int fp8_call(const kvs_geometry* g, const kvs_paged_cache* cache, const kvs_requ
             // where a whole-GPU launch per group displaces that compute, so it takes the
             // host-link store cap (exposed store time per 8B prefill: 7.7 ms uncapped,
             // 2.1 ms at 32 CTAs).
-            const int grid = cap ? cap : retrieve ? 2 * st.hostlink_ctas : layers_per_step > 0 ? st.store_ctas : 0;
+            // KVS_F_FEW_SMS: the staged kernel on the BF16 staged kernel's cap (each of its
+            // CTAs holds 112 KiB of codes, about what a BF16 staged CTA holds).
+            const int grid = cap ? cap : few ? st.few_sm_ctas : retrieve ? 2 * st.hostlink_ctas
+                           : layers_per_step > 0 ? st.store_ctas : 0;
             rc = run(f, grid, false);
             if (rc) return rc;
         }

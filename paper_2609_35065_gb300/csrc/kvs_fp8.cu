@@ -65,15 +65,23 @@ struct Fp8Piece {
 
 // Piece q -> addresses; false for pieces with nothing to move.  Runs are
 // (entry, plane, block) as for BF16 copies; a run holds ntok rows of H*D codes.
+__device__ __forceinline__ uint32_t fp8_div(uint32_t n, uint32_t m, uint32_t p) {
+    return (uint32_t)(((uint64_t)n * m) >> p);
+}
+
+// FAST: the reciprocal divisions (persistent kernels decode a piece per loop
+// trip); the one-piece-per-CTA kernel keeps plain divisions and per-vector head indices,
+// which holds it at fewer registers.
+template <bool FAST = true>
 __device__ __forceinline__ bool fp8_piece(const Fp8Job& f, uint32_t q, Fp8Piece& pc) {
     const Job& j = f.job;
     const uint32_t hd = f.heads * f.head_dim;
-    const uint32_t run = q / j.pieces_per_run;
-    const uint32_t k = q - run * j.pieces_per_run;
     const uint32_t per_entry = j.num_planes * j.blocks_per_chunk;
-    const uint32_t e = run / per_entry;
+    const uint32_t run = FAST ? fp8_div(q, f.ppr_m, f.ppr_p) : q / j.pieces_per_run;
+    const uint32_t k = q - run * j.pieces_per_run;
+    const uint32_t e = FAST ? fp8_div(run, f.pe_m, f.pe_p) : run / per_entry;
     const uint32_t rem = run - e * per_entry;
-    const uint32_t pr = rem / j.blocks_per_chunk;
+    const uint32_t pr = FAST ? fp8_div(rem, f.bpc_m, f.bpc_p) : rem / j.blocks_per_chunk;
     const uint32_t i = rem - pr * j.blocks_per_chunk;
     const uint32_t p = j.plane_begin + pr;
     const int32_t blk = __ldg(j.blocks + (size_t)(j.entry_base + e) * j.blocks_per_chunk + i);
@@ -150,8 +158,22 @@ __device__ __forceinline__ void rt_load(const Fp8Job& f, const Fp8Piece& pc, RtR
 
 // Publishes the piece's scales in shared memory (after every thread has finished
 // with the previous piece's), then converts and stores this thread's vectors.
-__device__ __forceinline__ void rt_store(const Fp8Job& f, const Fp8Piece& pc, const RtRegs& r, float* sm_scale) {
+// Head of this thread's vector v of a piece: when pieces start at token rows
+// and a row's vpr vectors divide the CTA's thread count T, vector tid + u*T
+// is always in head (tid % vpr) / vph, computed once per thread (`h_fixed`).
+__device__ __forceinline__ uint32_t fp8_fixed_head(const Fp8Job& f, uint32_t T) {
     const uint32_t vph = f.head_dim / 16, vpr = f.heads * vph;
+    return (f.rows_whole && T % vpr == 0) ? (threadIdx.x % vpr) / vph : 0xFFFFFFFFu;
+}
+
+__device__ __forceinline__ uint32_t fp8_head(const Fp8Job& f, const Fp8Piece& pc, uint32_t v, uint32_t h_fixed) {
+    if (h_fixed != 0xFFFFFFFFu) return h_fixed;
+    const uint32_t vph = f.head_dim / 16, vpr = f.heads * vph;
+    return ((pc.vec0 + v) % vpr) / vph;
+}
+
+__device__ __forceinline__ void rt_store(const Fp8Job& f, const Fp8Piece& pc, const RtRegs& r, float* sm_scale,
+                                         uint32_t h_fixed) {
     const uint32_t nv = pc.len / 16;
     __syncthreads();
     if (threadIdx.x < f.heads) sm_scale[threadIdx.x] = r.s;
@@ -161,7 +183,7 @@ __device__ __forceinline__ void rt_store(const Fp8Job& f, const Fp8Piece& pc, co
         const uint32_t v = threadIdx.x + u * kRtThreads;
         if (v < nv) {
             uint4 lo, hi;
-            dequant16(r.c[u], sm_scale[((pc.vec0 + v) % vpr) / vph], lo, hi);
+            dequant16(r.c[u], sm_scale[fp8_head(f, pc, v, h_fixed)], lo, hi);
             st_cs16(pc.out + (uint64_t)v * 32, lo);
             st_cs16(pc.out + (uint64_t)v * 32 + 16, hi);
         }
@@ -181,6 +203,7 @@ __device__ __forceinline__ bool rt_next(const Fp8Job& f, uint32_t n, uint32_t& q
 // depends only on blockIdx), so the barriers in rt_store are reached by all.
 __global__ void __launch_bounds__(kRtThreads) kvs_fp8_retrieve_kernel(const Fp8Job f, uint32_t num_pieces) {
     __shared__ float sm_scale[kFp8MaxHeads];
+    const uint32_t h_fixed = fp8_fixed_head(f, kRtThreads);
     RtRegs ra, rb;
     Fp8Piece pa, pb;
     uint32_t q = blockIdx.x;
@@ -189,11 +212,11 @@ __global__ void __launch_bounds__(kRtThreads) kvs_fp8_retrieve_kernel(const Fp8J
     while (ha) {
         const bool hb = rt_next(f, num_pieces, q, pb);
         if (hb) rt_load(f, pb, rb);
-        rt_store(f, pa, ra, sm_scale);
+        rt_store(f, pa, ra, sm_scale, h_fixed);
         if (!hb) break;
         ha = rt_next(f, num_pieces, q, pa);
         if (ha) rt_load(f, pa, ra);
-        rt_store(f, pb, rb, sm_scale);
+        rt_store(f, pb, rb, sm_scale, h_fixed);
     }
 }
 
@@ -204,10 +227,153 @@ __global__ void __launch_bounds__(kRtThreads) kvs_fp8_retrieve_kernel(const Fp8J
 __global__ void __launch_bounds__(kRtThreads, 8) kvs_fp8_retrieve_piece_kernel(const Fp8Job f) {
     __shared__ float sm_scale[kFp8MaxHeads];
     Fp8Piece pc;
-    if (!fp8_piece(f, blockIdx.x, pc)) return;         // uniform across the CTA
+    if (!fp8_piece<false>(f, blockIdx.x, pc)) return;  // uniform across the CTA
     RtRegs r;
     rt_load(f, pc, r);
-    rt_store(f, pc, r, sm_scale);
+    rt_store(f, pc, r, sm_scale, 0xFFFFFFFFu);
+}
+
+// Few-SM flavour of the host-chunk retrieval (KVS_F_FEW_SMS): the scheme of
+// the host-link BF16 staged kernel.  A 256-thread CTA keeps seven 16 KiB pieces
+// of codes in flight: two in registers and five in shared memory, where each
+// thread copies, with cp.async, its own 16-code vectors and the binary32 scale
+// of each vector's head into slots that only it reads back (no CTA barrier).
+// 100 KiB of shared memory per CTA, two CTAs per SM: 224 KiB of codes in flight
+// per SM, where kvs_fp8_retrieve_kernel holds 128 KiB.  Piece i of a CTA lives
+// in slot i % 7; pieces come in grid-stride order, so once a slot finds none
+// left, neither does any slot after it.
+constexpr int kFsThreads = 256;
+constexpr int kFsVec = kFp8PieceCodes / 16 / kFsThreads;             // vectors per thread per piece
+constexpr int kFsRegPieces = 2;
+constexpr int kFsSmemPieces = 5;
+constexpr int kFsSlots = kFsRegPieces + kFsSmemPieces;
+constexpr uint32_t kFsSlotBytes = kFp8PieceCodes + kFp8PieceCodes / 16 * 4;   // codes + a scale per vector
+constexpr uint32_t kFsSmemBytes = kFsSmemPieces * kFsSlotBytes;
+static_assert(kFsVec * kFsThreads * 16 == kFp8PieceCodes, "a piece is one vector set per CTA");
+
+__device__ __forceinline__ void fs_cp16(uint32_t dst, uint64_t src) {
+    asm volatile("cp.async.cg.shared.global [%0], [%1], 16;" :: "r"(dst), "l"(src) : "memory");
+}
+
+__device__ __forceinline__ void fs_cp4(uint32_t dst, uint64_t src) {
+    asm volatile("cp.async.ca.shared.global [%0], [%1], 4;" :: "r"(dst), "l"(src) : "memory");
+}
+
+__device__ __forceinline__ void fs_commit() {
+    asm volatile("cp.async.commit_group;" ::: "memory");
+}
+
+template <int N>
+__device__ __forceinline__ void fs_wait() {
+    asm volatile("cp.async.wait_group %0;" :: "n"(N) : "memory");
+}
+
+// Scale address of vector v of piece pc (its head's binary32 scale).
+__device__ __forceinline__ uint64_t fs_scale_addr(const Fp8Job& f, const Fp8Piece& pc, uint32_t v, uint32_t h_fixed) {
+    return pc.scales + (uint64_t)fp8_head(f, pc, v, h_fixed) * 4;
+}
+
+struct FsRegs {
+    uint4 c[kFsVec];
+    float s[kFsVec];
+};
+
+__device__ __forceinline__ void fs_load_regs(const Fp8Job& f, const Fp8Piece& pc, FsRegs& r, uint32_t h_fixed) {
+    const uint32_t nv = pc.len / 16;
+#pragma unroll
+    for (int u = 0; u < kFsVec; ++u) {
+        const uint32_t v = threadIdx.x + u * kFsThreads;
+        if (v < nv) {
+            r.c[u] = ld_nc16(pc.codes + (uint64_t)v * 16);
+            r.s[u] = __ldg(reinterpret_cast<const float*>(fs_scale_addr(f, pc, v, h_fixed)));
+        }
+    }
+}
+
+__device__ __forceinline__ void fs_store_regs(const Fp8Piece& pc, const FsRegs& r) {
+    const uint32_t nv = pc.len / 16;
+#pragma unroll
+    for (int u = 0; u < kFsVec; ++u) {
+        const uint32_t v = threadIdx.x + u * kFsThreads;
+        if (v < nv) {
+            uint4 lo, hi;
+            dequant16(r.c[u], r.s[u], lo, hi);
+            st_cs16(pc.out + (uint64_t)v * 32, lo);
+            st_cs16(pc.out + (uint64_t)v * 32 + 16, hi);
+        }
+    }
+}
+
+// Slot layout: codes of vector v at v * 16, its scale at kFp8PieceCodes + v * 4.
+__device__ __forceinline__ void fs_stage(const Fp8Job& f, const Fp8Piece& pc, uint32_t slot, uint32_t h_fixed) {
+    const uint32_t nv = pc.len / 16;
+#pragma unroll
+    for (int u = 0; u < kFsVec; ++u) {
+        const uint32_t v = threadIdx.x + u * kFsThreads;
+        if (v < nv) {
+            fs_cp16(slot + v * 16, pc.codes + (uint64_t)v * 16);
+            fs_cp4(slot + kFp8PieceCodes + v * 4, fs_scale_addr(f, pc, v, h_fixed));
+        }
+    }
+}
+
+__device__ __forceinline__ void fs_unstage(const Fp8Piece& pc, uint32_t slot) {
+    const uint32_t nv = pc.len / 16;
+#pragma unroll
+    for (int u = 0; u < kFsVec; ++u) {
+        const uint32_t v = threadIdx.x + u * kFsThreads;
+        if (v < nv) {
+            uint4 c;
+            float sc;
+            asm volatile("ld.shared.v4.u32 {%0,%1,%2,%3}, [%4];"
+                         : "=r"(c.x), "=r"(c.y), "=r"(c.z), "=r"(c.w) : "r"(slot + v * 16));
+            asm volatile("ld.shared.f32 %0, [%1];" : "=f"(sc) : "r"(slot + kFp8PieceCodes + v * 4));
+            uint4 lo, hi;
+            dequant16(c, sc, lo, hi);
+            st_cs16(pc.out + (uint64_t)v * 32, lo);
+            st_cs16(pc.out + (uint64_t)v * 32 + 16, hi);
+        }
+    }
+}
+
+__global__ void __launch_bounds__(kFsThreads, 2) kvs_fp8_retrieve_staged_kernel(const Fp8Job f, uint32_t num_pieces) {
+    extern __shared__ __align__(128) uint8_t fs_smem[];
+    const uint32_t base = smem_u32(fs_smem);
+    const uint32_t h_fixed = fp8_fixed_head(f, kFsThreads);
+    FsRegs r[kFsRegPieces];
+    Fp8Piece pc[kFsSlots];
+    bool has[kFsSlots];
+    uint32_t q = blockIdx.x;
+    // fill slot s with the CTA's next piece; a shared-memory slot always commits
+    // one group (empty past the end), so wait_group counts pieces
+    auto fill = [&](int s) {
+        has[s] = rt_next(f, num_pieces, q, pc[s]);
+        if (s < kFsRegPieces) {
+            if (has[s]) fs_load_regs(f, pc[s], r[s < kFsRegPieces ? s : 0], h_fixed);
+        } else {
+            if (has[s]) fs_stage(f, pc[s], base + (s - kFsRegPieces) * kFsSlotBytes, h_fixed);
+            fs_commit();
+        }
+    };
+#pragma unroll
+    for (int s = 0; s < kFsSlots; ++s) fill(s);
+    bool more = true;
+    while (more) {
+#pragma unroll
+        for (int s = 0; s < kFsSlots; ++s) {
+            if (more && !has[s]) more = false;
+            if (more) {
+                if (s < kFsRegPieces) {
+                    fs_store_regs(pc[s], r[s < kFsRegPieces ? s : 0]);
+                } else {
+                    fs_wait<kFsSmemPieces - 1>();    // the younger shared-memory pieces may be in flight
+                    fs_unstage(pc[s], base + (s - kFsRegPieces) * kFsSlotBytes);
+                }
+                fill(s);
+            }
+        }
+    }
+    fs_wait<0>();
 }
 
 // ---------------------------------------------------------------------------
@@ -684,6 +850,7 @@ __global__ void __launch_bounds__(kStThreads) kvs_fp8_store_kernel(const Fp8Job 
 int g_sms = 0;
 constexpr int kMaxDev = 64;
 bool g_sg_attr[kMaxDev];                 // dynamic shared memory limit of the staged store raised
+bool g_fs_attr[kMaxDev];                 // ... of the few-SM retrieval
 
 int sm_count() {
     if (g_sms == 0) {
@@ -710,6 +877,27 @@ cudaError_t launch_fp8_retrieve(const Fp8Job& fj, int grid, cudaStream_t s) {
     if (grid <= 0 || grid > full) grid = full;
     if ((uint64_t)grid > n) grid = (int)n;
     kvs_fp8_retrieve_kernel<<<grid, kRtThreads, 0, s>>>(fj, (uint32_t)n);
+    return cudaGetLastError();
+}
+
+cudaError_t launch_fp8_retrieve_staged(const Fp8Job& fj, int grid, cudaStream_t s) {
+    const uint64_t n = fj.job.num_pieces;
+    if (n == 0) return cudaSuccess;
+    int dev = 0;
+    cudaGetDevice(&dev);
+    if (dev < 0 || dev >= kMaxDev) dev = 0;
+    if (!g_fs_attr[dev]) {
+        cudaError_t e = cudaFuncSetAttribute(kvs_fp8_retrieve_staged_kernel,
+                                             cudaFuncAttributeMaxDynamicSharedMemorySize, (int)kFsSmemBytes);
+        if (e == cudaSuccess)
+            e = cudaFuncSetAttribute(kvs_fp8_retrieve_staged_kernel, cudaFuncAttributePreferredSharedMemoryCarveout, 100);
+        if (e != cudaSuccess) return e;
+        g_fs_attr[dev] = true;
+    }
+    const int full = sm_count() * 2;
+    if (grid <= 0 || grid > full) grid = full;
+    if ((uint64_t)grid > n) grid = (int)n;
+    kvs_fp8_retrieve_staged_kernel<<<grid, kFsThreads, kFsSmemBytes, s>>>(fj, (uint32_t)n);
     return cudaGetLastError();
 }
 

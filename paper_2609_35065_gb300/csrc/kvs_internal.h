@@ -87,6 +87,11 @@ struct Fp8Job {
     uint32_t head_dim;           // D, a multiple of 16
     uint32_t scale_bytes;        // bytes of the scale block, a multiple of 256
     uint32_t block_magic;        // floor(2^32 / B) + 1: floor(i / B) = umulhi(i, magic) for i, B < 2^16
+    // Piece decode by round-up reciprocals: floor(n / d) = (n * m) >> p for n < 2^31
+    // (p = 31 + ceil(log2 d), m = ceil(2^p / d)), d = pieces per run, runs per
+    // entry (num_planes * blocks_per_chunk) and blocks per chunk.
+    uint32_t ppr_m, ppr_p, pe_m, pe_p, bpc_m, bpc_p;
+    uint32_t rows_whole;         // 1 when every piece starts at a token row (H*D/16 divides 1024)
 };
 constexpr uint32_t kFp8MaxHeads = 128;
 // Retrieval: a persistent grid of `grid` CTAs (<= 0: fill the GPU) over pieces of at
@@ -94,6 +99,10 @@ constexpr uint32_t kFp8MaxHeads = 128;
 // (HBM sources).  The number of pieces is in job.num_pieces.
 constexpr int kFp8PerPiece = -1;
 cudaError_t launch_fp8_retrieve(const Fp8Job& fj, int grid, cudaStream_t s);
+// Retrieval of host chunks with more codes in flight per SM (two pieces in
+// registers and five in shared memory per 256 threads, two CTAs per SM), for
+// GPUs that run other kernels meanwhile (KVS_F_FEW_SMS); `grid` <= 0: 2 per SM.
+cudaError_t launch_fp8_retrieve_staged(const Fp8Job& fj, int grid, cudaStream_t s);
 // Store-back: one CTA per (entry, plane, head) in a single pass when a head's
 // chunk_tokens x head_dim elements fit the CTA's registers, else one CTA per
 // (entry, plane) in two passes; a grid-stride loop over them with `grid` > 0.

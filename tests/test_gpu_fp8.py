@@ -326,3 +326,41 @@ def test_fp8_store_nan_without_infinity(store_residency):
     _store(buf)
     torch.cuda.synchronize()
     gc.check_store_fp8(buf)
+
+
+@pytest.mark.parametrize("cap", [0, 1, 6], ids=["default_grid", "1_cta", "6_ctas"])
+def test_fp8_few_sms_retrieval(cap):
+    """KVS_F_FEW_SMS with fp8 chunks (two pieces of codes in registers and five in shared
+    memory, scales copied per vector): the 8B batch shape (2 requests) and a mixed, ragged
+    shape with an odd head count, every element against the oracle; stores ignore the flag."""
+    flags = kvs.KVS_F_FEW_SMS | kvs.KVS_F_VALIDATE | kvs.KVS_F_MAX_CTAS(cap)
+    for w in (synth.llama8b(requests=2, num_blocks=1024),
+              synth.custom(3, 5, 48, 16, 64, 300, [700, 520, 400], [640, 448, 320], seed=cap,
+                           residency=["host", "device", "host"], firsts=[0, 64, 0], store_tokens=[0, 0, 0])):
+        buf = buffers.allocate_fp8(w)
+        _retrieve(buf, flags)
+        torch.cuda.synchronize()
+        gc.check_retrieve_fp8(buf)
+
+
+def test_fp8_few_sms_layer_groups():
+    """Layer-wise fp8 retrieval on the few-SM kernel: each group's event fires after exactly
+    the oracle's planes of that group."""
+    w = synth.custom(4, 8, 128, 16, 256, 200, [1024, 768], [1024, 768], seed=21)
+    g = w.geom
+    buf = buffers.allocate_fp8(w)
+    events = [torch.cuda.Event() for _ in range(2)]
+    copier, consumer = torch.cuda.Stream(), torch.cuda.Stream()
+    kvs.kvs_retrieve_fp8_layers(g, buf.plane_ptrs, w.num_blocks, buf.requests, 2, events, copier, kvs.KVS_F_FEW_SMS)
+    snaps = []
+    for k, ev in enumerate(events):
+        consumer.wait_event(ev)
+        with torch.cuda.stream(consumer):
+            snaps.append(buf.planes[4 * k:4 * k + 4].clone())
+    torch.cuda.synchronize()
+    assert kvs.kvs_check_errors(None) == kvs.KVS_OK
+    chunks_np = [[gc._np(t) for t in mine] for mine in buf.chunks]
+    for k, snap in enumerate(snaps):
+        for i in range(4):
+            want = gc.expected_plane_fp8(buf, 4 * k + i, chunks_np)
+            assert np.array_equal(snap[i].cpu().numpy().view(np.uint16), want), (k, i)

@@ -67,7 +67,8 @@ def test_calls_from_several_host_threads():
         gc.check_retrieve(b)
 
 
-def test_retrieval_beside_a_gemm_loop_is_exact():
+@pytest.mark.parametrize("flags", [0, kvs.KVS_F_FEW_SMS], ids=["default", "few_sms"])
+def test_retrieval_beside_a_gemm_loop_is_exact(flags):
     buf = buffers.allocate(synth.llama8b(requests=2, num_blocks=1024))
     w = buf.workload
     side = torch.cuda.Stream(priority=-1)
@@ -75,7 +76,7 @@ def test_retrieval_beside_a_gemm_loop_is_exact():
     c = torch.empty_like(a)
     for _ in range(20):
         torch.matmul(a, a, out=c)                           # queued on the main stream
-    kvs.kvs_retrieve(w.geom, buf.plane_ptrs, w.num_blocks, buf.requests, side, 0)
+    kvs.kvs_retrieve(w.geom, buf.plane_ptrs, w.num_blocks, buf.requests, side, flags)
     for _ in range(20):
         torch.matmul(a, a, out=c)
     torch.cuda.synchronize()
