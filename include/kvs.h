@@ -313,7 +313,7 @@ typedef struct kvs_bw_report {
     int32_t chosen_kernel_device;  /* KVS_KERNEL_* used for device-resident chunks         */
     int32_t num_sms;
     int32_t hostlink_ctas;         /* CTAs given to host-link retrieval kernels (0 = all):
-                                      4 x the smallest probed grid within 0.5% of the best
+                                      4 x the smallest probed grid within 1% of the best
                                       rate, so that kernels on other streams keep most SMs
                                       (before any kvs_query_bw: one per 3 SMs)            */
     int32_t store_ctas;            /* the same for host-link store kernels                 */

@@ -1129,7 +1129,7 @@ int query_bw(DevState& st, kvs_bw_report* out, cudaStream_t s, int64_t probe_byt
         cleanup();
         return rc;
     }
-    // Host-link grid cap: four times the smallest grid within 0.5% of the best
+    // Host-link grid cap: four times the smallest grid within 1% of the best
     // rate on an idle GPU.  A grid that fills every SM buys nothing once the
     // link is saturated and starves kernels on other streams; the margin covers
     // the longer load latency when other kernels load the GPU (measured beside
@@ -1148,7 +1148,7 @@ int query_bw(DevState& st, kvs_bw_report* out, cudaStream_t s, int64_t probe_byt
             }
             int pick = 0;
             for (int k = 0; k < ncand; ++k)
-                if (gb[dir][k] >= 0.995 * best) { pick = cand[k]; break; }
+                if (gb[dir][k] >= 0.99 * best) { pick = cand[k]; break; }
             pick *= 4;
             if (pick >= full) pick = 0;
             if (dir == 0) rep.hostlink_ctas = pick; else rep.store_ctas = pick;
