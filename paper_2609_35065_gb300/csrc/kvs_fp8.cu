@@ -847,19 +847,21 @@ __global__ void __launch_bounds__(kStThreads) kvs_fp8_store_kernel(const Fp8Job 
     }
 }
 
-int g_sms = 0;
 constexpr int kMaxDev = 64;
+int g_sms[kMaxDev];                      // SM count per device
 bool g_sg_attr[kMaxDev];                 // dynamic shared memory limit of the staged store raised
 bool g_fs_attr[kMaxDev];                 // ... of the few-SM retrieval
 
 int sm_count() {
-    if (g_sms == 0) {
-        int dev = 0, n = 0;
-        cudaGetDevice(&dev);
+    int dev = 0;
+    cudaGetDevice(&dev);
+    if (dev < 0 || dev >= kMaxDev) dev = 0;
+    if (g_sms[dev] == 0) {
+        int n = 0;
         cudaDeviceGetAttribute(&n, cudaDevAttrMultiProcessorCount, dev);
-        g_sms = n > 0 ? n : 1;
+        g_sms[dev] = n > 0 ? n : 1;
     }
-    return g_sms;
+    return g_sms[dev];
 }
 
 }  // namespace
