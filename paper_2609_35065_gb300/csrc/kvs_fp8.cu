@@ -581,14 +581,17 @@ __device__ __forceinline__ void sts16_zero(uint32_t a) {
     asm volatile("st.shared.v4.u32 [%0], {%1,%1,%1,%1};" :: "r"(a), "r"(0u) : "memory");
 }
 
-// Two BF16 (one word) times `inv` -> two E4M3 codes, with one packed binary32
-// multiply (sm_100+; each lane rounded to nearest like __fmul_rn).
+// Two BF16 (one word) times `inv` -> two E4M3 codes: two binary32 multiplies
+// rounded to nearest, then one saturating nearest-even pair conversion (the
+// high element goes to the high byte).  (A packed f32x2 multiply measured 0.5%
+// slower here.)
 __device__ __forceinline__ uint32_t e4m3x2_of_pk(uint32_t w, uint64_t inv2) {
-    const uint64_t x2 = ((uint64_t)(w & 0xFFFF0000u) << 32) | (uint64_t)(w << 16);
-    uint64_t q2;
-    asm("mul.rn.f32x2 %0, %1, %2;" : "=l"(q2) : "l"(x2), "l"(inv2));
-    return (uint32_t)__nv_cvt_float2_to_fp8x2(
-        make_float2(__uint_as_float((uint32_t)q2), __uint_as_float((uint32_t)(q2 >> 32))), __NV_SATFINITE, __NV_E4M3);
+    const float inv = __uint_as_float((uint32_t)inv2);
+    const float lo = __fmul_rn(__uint_as_float(w << 16), inv), hi = __fmul_rn(__uint_as_float(w & 0xFFFF0000u), inv);
+    uint32_t r;
+    asm("{\n\t.reg .b16 t;\n\tcvt.rn.satfinite.e4m3x2.f32 t, %1, %2;\n\tcvt.u32.u16 %0, t;\n\t}"
+        : "=r"(r) : "f"(hi), "f"(lo));
+    return r;
 }
 
 __device__ __forceinline__ uint2 quant8_pk(const uint4& a, uint64_t inv2) {
