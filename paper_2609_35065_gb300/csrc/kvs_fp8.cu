@@ -29,7 +29,9 @@
 // loads are in flight while the current one is converted and stored.  The H
 // scales of a piece's plane are loaded once per piece by H threads (one 4-byte
 // load each, beside the codes) and shared through shared memory, instead of
-// one scale load per vector; HBM chunks run one CTA per piece instead.
+// one scale load per vector; HBM chunks run one CTA per piece instead, and
+// KVS_F_FEW_SMS runs a kernel that also stages pieces in shared memory so
+// that fewer SMs hold the link beside other kernels.
 // Store-back to pinned host runs one 256-thread CTA per (chunk, plane, head):
 // the head's BF16 elements are loaded into registers at once, reduced to the
 // amax and quantised from registers (heads too large for that take a two-pass
