@@ -364,3 +364,18 @@ def test_fp8_few_sms_layer_groups():
         for i in range(4):
             want = gc.expected_plane_fp8(buf, 4 * k + i, chunks_np)
             assert np.array_equal(snap[i].cpu().numpy().view(np.uint16), want), (k, i)
+
+
+def test_fp8_llama8b_batch_few_sms():
+    """The full 8B batch (128 fp8 chunks, 2 GiB of codes in pinned host memory) retrieved
+    with KVS_F_FEW_SMS on its default cap after kvs_query_bw, as the overlap benchmark runs
+    it; every plane against the oracle."""
+    s = torch.cuda.Stream()
+    kvs.kvs_query_bw(s, 256 << 20)
+    w = synth.llama8b()
+    buf = buffers.allocate_fp8(w)
+    kvs.kvs_retrieve_fp8(w.geom, buf.plane_ptrs, w.num_blocks, buf.requests, s, kvs.KVS_F_FEW_SMS)
+    s.synchronize()
+    assert kvs.kvs_check_errors(s) == kvs.KVS_OK
+    gc.check_retrieve_fp8(buf)
+    kvs.kvs_shutdown()

@@ -110,10 +110,12 @@ def test_qwen14b_store_to_hbm_destination_hbmcopy_path():
     gc.free(buf)
 
 
-@pytest.mark.parametrize("frac", [0.25, 0.5], ids=["25pct", "50pct"])
-def test_llama70b_partial_buffer_refilled_between_passes(frac):
+@pytest.mark.parametrize("frac,flags", [(0.25, 0), (0.5, 0), (0.25, kvs.KVS_F_FEW_SMS)],
+                         ids=["25pct", "50pct", "25pct_few_sms"])
+def test_llama70b_partial_buffer_refilled_between_passes(frac, flags):
     """Pinned fast-tier buffer holds 25% (4 passes of one request) or 50% (2 passes of two
-    requests) of the batch, refilled in between; every pass is one call."""
+    requests) of the batch, refilled in between; every pass is one call (with
+    KVS_F_FEW_SMS: the staged kernel on its cap, as the overlap benchmark runs it)."""
     w = synth.llama70b(buffer_frac=frac)
     g = w.geom
     per_tok = 2 * g.layers * g.row_elems
@@ -138,7 +140,7 @@ def test_llama70b_partial_buffer_refilled_between_passes(frac):
                       for j in range(r.matched_tokens // 256)]
             reqs.append(kvs.RequestArg(r.block_table, [kvs.ChunkArg(c, 256) for c in chunks]))
             host_copies.append([c.numpy().copy().view(np.uint16) for c in chunks])
-        kvs.kvs_retrieve(g, ptrs, w.num_blocks, reqs, None, kvs.KVS_F_VALIDATE)
+        kvs.kvs_retrieve(g, ptrs, w.num_blocks, reqs, None, kvs.KVS_F_VALIDATE | flags)
         torch.cuda.synchronize()
     fake = buffers.Buffers(w, planes, [], [], [], [])
     gc.check_retrieve(fake, chunks_np=host_copies)
