@@ -355,8 +355,8 @@ int kvs_get_choice(kvs_bw_report* out);
  * candidate produces the same result, so the call's copy is done when
  * kvs_tune returns (the stream is synchronised).  KVS_F_MAX_CTAS(n) caps the
  * HOSTLINK candidate's grid (and becomes the host-link cap of that direction
- * if it wins); KVS_F_VALIDATE is honoured on the untimed runs; FORCE flags are
- * KVS_ERR_INVALID_ARG.  When the call holds device-resident chunks, those
+ * if it wins); KVS_F_VALIDATE is honoured on the untimed runs; FORCE, layer,
+ * KVS_F_FEW_SMS and KVS_F_PREFETCH_L2 flags are KVS_ERR_INVALID_ARG.  When the call holds device-resident chunks, those
  * chunks alone are then timed with the LDG and the TMA kernel (TMA only for
  * 16-byte aligned data), each chunk as a request of its own, and the faster
  * kernel becomes the default for device chunks.  A call with no chunk of a

@@ -1204,9 +1204,6 @@ int query_bw(DevState& st, kvs_bw_report* out, cudaStream_t s, int64_t probe_byt
 
 int tune(DevState& st, const kvs_geometry* g, const kvs_paged_cache* cache, const kvs_request* reqs,
          int32_t nreq, cudaStream_t s, uint32_t flags, int32_t direction, int32_t reps, kvs_tune_report* out) {
-    const uint32_t forced = KVS_F_FORCE_HOSTLINK | KVS_F_FORCE_HBMCOPY | KVS_F_FORCE_DMA | KVS_F_FORCE_LDG |
-                            KVS_F_FORCE_TMA | KVS_F_LAYER_LAUNCHES | KVS_F_LAYER_SIGNAL;
-    if (flags & forced) return fail(KVS_ERR_INVALID_ARG, "kvs_tune chooses the variant: no FORCE or layer flags");
     if (direction != KVS_DIR_RETRIEVE && direction != KVS_DIR_STORE)
         return fail(KVS_ERR_INVALID_ARG, "direction must be KVS_DIR_RETRIEVE or KVS_DIR_STORE");
     if (reps < 1 || reps > 1000) return fail(KVS_ERR_INVALID_ARG, "reps must be in [1, 1000]");
@@ -1405,6 +1402,13 @@ int kvs_tune(const kvs_geometry* geom, const kvs_paged_cache* cache, const kvs_r
     if (direction != KVS_DIR_RETRIEVE && direction != KVS_DIR_STORE)
         return fail(KVS_ERR_INVALID_ARG, "direction must be KVS_DIR_RETRIEVE or KVS_DIR_STORE");
     if (reps < 1 || reps > 1000) return fail(KVS_ERR_INVALID_ARG, "reps must be in [1, 1000]");
+    // kernel choices that kvs_tune's candidates would not carry: refused rather than ignored
+    const uint32_t forced = KVS_F_FORCE_HOSTLINK | KVS_F_FORCE_HBMCOPY | KVS_F_FORCE_DMA | KVS_F_FORCE_LDG |
+                            KVS_F_FORCE_TMA | KVS_F_LAYER_LAUNCHES | KVS_F_LAYER_SIGNAL | KVS_F_FEW_SMS |
+                            KVS_F_PREFETCH_L2;
+    if (flags & forced)
+        return fail(KVS_ERR_INVALID_ARG, "kvs_tune chooses the variant: no FORCE, layer, KVS_F_FEW_SMS or "
+                    "KVS_F_PREFETCH_L2 flags");
     Plan pl;
     int rc = validate_call(geom, cache, requests, num_requests, pl);      // before any device state
     if (rc) return rc;

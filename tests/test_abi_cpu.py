@@ -244,3 +244,13 @@ def test_the_abi_from_plain_c(tmp_path):
     assert out.returncode == 0, (out.returncode, out.stderr)
     assert out.stdout.strip() == "ok"
 
+
+
+@pytest.mark.parametrize("flags", [kvs.KVS_F_FORCE_HOSTLINK, kvs.KVS_F_FEW_SMS, kvs.KVS_F_PREFETCH_L2,
+                                   kvs.KVS_F_LAYER_SIGNAL], ids=["force", "few_sms", "prefetch_l2", "layer"])
+def test_tune_refuses_kernel_choice_flags_before_device_work(flags):
+    """kvs_tune picks the variant itself: flags that would choose a kernel for it are
+    refused on the host, with no GPU (its candidates would not carry them)."""
+    with pytest.raises(kvs.KvsError) as ei:
+        kvs.kvs_tune(G, _planes(), 8, [_req()], None, flags, kvs.KVS_DIR_RETRIEVE, 1)
+    assert ei.value.code == kvs.KVS_ERR_INVALID_ARG

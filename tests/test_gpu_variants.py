@@ -146,7 +146,8 @@ def test_tune_choice_follows_the_measurement(direction):
 def test_tune_argument_checks():
     buf = buffers.allocate(synth.tiny())
     w = buf.workload
-    for flags, direction, reps in [(kvs.KVS_F_FORCE_DMA, 0, 1), (0, 2, 1), (0, 0, 0)]:
+    for flags, direction, reps in [(kvs.KVS_F_FORCE_DMA, 0, 1), (0, 2, 1), (0, 0, 0), (kvs.KVS_F_FEW_SMS, 0, 1),
+                                   (kvs.KVS_F_PREFETCH_L2, 0, 1)]:
         with pytest.raises(kvs.KvsError) as ei:
             kvs.kvs_tune(w.geom, buf.plane_ptrs, w.num_blocks, buf.requests, None, flags, direction, reps)
         assert ei.value.code == kvs.KVS_ERR_INVALID_ARG
