@@ -702,15 +702,20 @@ cudaError_t launch_link_prefetch(const Job& job, int grid, cudaStream_t s) {
     return cudaGetLastError();
 }
 
+// Raises the kernel's dynamic shared-memory limit on the current device (once
+// per device) and returns its resident CTAs per SM.
+int g_staged_per_sm[kMaxDevices];
+
 int link_staged_ctas_per_sm() {
-    static int n = 0;
-    if (n == 0) {
+    const int dev = current_device();
+    if (g_staged_per_sm[dev] == 0) {
         cudaFuncSetAttribute(kvs_link_staged_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)kStagedSmemBytes);
         cudaFuncSetAttribute(kvs_link_staged_kernel, cudaFuncAttributePreferredSharedMemoryCarveout, 100);
+        int n = 0;
         cudaOccupancyMaxActiveBlocksPerMultiprocessor(&n, kvs_link_staged_kernel, kLdgThreads, kStagedSmemBytes);
-        if (n <= 0) n = 1;
+        g_staged_per_sm[dev] = n > 0 ? n : 1;
     }
-    return n;
+    return g_staged_per_sm[dev];
 }
 
 cudaError_t launch_link_staged(const Job& job, int grid, cudaStream_t s) {
